@@ -1,0 +1,317 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix (no GPU).
+
+Each test checks the oracle against something other than itself: a worked example
+derived by hand, a closed form, an invariant of the method, or an independent
+library routine (torch / scipy) for a textbook primitive.
+"""
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as TF
+
+from oracle import cachedsearch_oracle as O
+from paper_2607_23159_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _tiny_model(blocks=2):
+    cfg = synth.replace_model(synth.TINY, blocks=blocks)
+    _, params = synth.make_params(cfg)
+    return cfg, O.DiT(cfg, params)
+
+
+def _read_golden(name):
+    out = {}
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            if line.startswith("#") or not line.strip():
+                continue
+            key, *vals = line.split()
+            out[key] = np.array([float(v) for v in vals])
+    return out
+
+
+# ---------------------------------------------------------------- sampler -----
+
+def test_time_grid_endpoints_and_spacing():
+    t = O.time_grid(50)
+    assert t[0] == 1.0 and t[-1] == 0.0 and len(t) == 51
+    assert np.all(np.diff(t) < 0)
+    np.testing.assert_allclose(np.diff(t), -1 / 50, rtol=0, atol=1e-15)
+
+
+def test_euler_linear_field_closed_form():
+    # v(x) = lam x  =>  x_{T+1} = prod_k (1 + h_k lam) x_1 exactly (Eq. euler)
+    lam, T = -0.7, 13
+    x1 = np.array([1.5, -2.0, 0.25])
+    x = O.rollout_uncached(x1, T, lambda x, t: lam * x)
+    t = O.time_grid(T)
+    np.testing.assert_allclose(x, np.prod(1 + np.diff(t) * lam) * x1, rtol=1e-14)
+
+
+def test_euler_constant_field_reaches_x1_minus_v():
+    # constant velocity c on the grid 1 -> 0: x_0 = x_1 - c (sum of steps is -1)
+    c = np.array([0.3, -1.1])
+    x = O.rollout_uncached(np.array([2.0, 5.0]), 7, lambda x, t: c)
+    np.testing.assert_allclose(x, np.array([2.0, 5.0]) - c, rtol=0, atol=1e-14)
+
+
+# --------------------------------------------------------------- cache rule ---
+
+def test_cache_rule_worked_example():
+    g = _read_golden("cache_rule_1d.txt")
+    xf, comp, acc = O.rollout(np.array([1.0]), 10, 0.25, 0, 0, lambda x, t: np.array([-1.0]))
+    np.testing.assert_array_equal(comp.astype(int), g["computed"].astype(int))
+    np.testing.assert_allclose(acc, g["accum_after_step"], rtol=0, atol=1e-12)
+    np.testing.assert_allclose(xf, g["x_final"], rtol=0, atol=1e-12)
+
+
+def test_tau_zero_is_uncached_sampling_bitwise():
+    # "off" mode recovers G exactly (Sec. 3.1 Properties; bit-exact no-cache control)
+    cfg, m = _tiny_model()
+    kv = m.text_kv(synth.text_context(cfg))
+    x1 = synth.initial_noise(cfg, [3])[0]
+    vel = lambda x, t: m.velocity(x, t, kv)
+    xc, comp, _ = O.rollout(x1, 10, 0.0, 1, 1, vel)
+    xu = O.rollout_uncached(x1, 10, vel)
+    assert comp.all()
+    assert np.array_equal(xc, xu)
+
+
+def test_huge_tau_skips_every_step_after_the_first_closed_form():
+    # K_w = K_c = 0: step 1 computes (empty cache), every later step skips.  With
+    # u_k = x_k + Delta a skip gives u_{k+1} = (1 + h_k) u_k, so
+    # x_{T+1} = -Delta + prod_{k>=2}(1 + h_k) (x_2 + Delta), Delta = v(x_1) - x_1.
+    cfg, m = _tiny_model()
+    kv = m.text_kv(synth.text_context(cfg))
+    x1 = synth.initial_noise(cfg, [1])[0].astype(np.float64)
+    T = 10
+    vel = lambda x, t: m.velocity(x, t, kv)
+    xf, comp, _ = O.rollout(x1, T, 1e30, 0, 0, vel)
+    assert comp[0] and not comp[1:].any()
+    t = O.time_grid(T)
+    v1 = m.velocity(x1, t[0], kv)
+    delta = v1 - x1
+    x2 = x1 + (t[1] - t[0]) * v1
+    expect = -delta + np.prod(1 + np.diff(t)[1:]) * (x2 + delta)
+    np.testing.assert_allclose(xf, expect, rtol=1e-12, atol=1e-12)
+
+
+def test_warmup_cooldown_windows_force_compute():
+    # v = 0 keeps x fixed, so the drift is 0 and every free step skips; only the
+    # warmup (k <= K_w) and cooldown (k > T - K_c) windows compute.
+    _, comp, _ = O.rollout(np.ones(4), 12, 0.1, 3, 2, lambda x, t: np.zeros(4))
+    assert comp.astype(int).tolist() == [1, 1, 1, 0, 0, 0, 0, 0, 0, 0, 1, 1]
+
+
+def test_forced_decision_replays_mask():
+    f = np.array([1, 0, 0, 1, 0, 1, 0, 0, 0, 1], bool)
+    _, comp, _ = O.rollout(np.array([1.0]), 10, 0.25, 0, 0, lambda x, t: np.array([-1.0]), f)
+    assert np.array_equal(comp, f)
+    with pytest.raises(ValueError):
+        O.rollout(np.array([1.0]), 3, 0.25, 0, 0, lambda x, t: x, np.array([0, 1, 1], bool))
+
+
+def test_search_step_equals_per_candidate_rollout():
+    # batched advance of N candidates = N independent rollouts (batch invariance)
+    cfg, m = _tiny_model()
+    kv = m.text_kv(synth.text_context(cfg))
+    x1s = synth.initial_noise(cfg, range(3)).astype(np.float64)
+    vel = lambda x, t: m.velocity(x, t, kv)
+    T = 6
+    states = [O.CacheState() for _ in range(3)]
+    xs = x1s.copy()
+    masks = []
+    for k in range(1, T + 1):
+        xs, skipped, _, _ = O.search_step(states, xs, k, T, 0.1, 1, 1, vel)
+        masks.append(~skipped)
+    for i in range(3):
+        xf, comp, _ = O.rollout(x1s[i], T, 0.1, 1, 1, vel)
+        assert np.array_equal(xf, xs[i])
+        assert np.array_equal(comp, np.array(masks)[:, i])
+
+
+def test_x0_estimate_score_on_last_step_is_final_latent_score():
+    cfg, m = _tiny_model()
+    kv = m.text_kv(synth.text_context(cfg))
+    x1s = synth.initial_noise(cfg, range(2)).astype(np.float64)
+    y = synth.target_latent(cfg)
+    vel = lambda x, t: m.velocity(x, t, kv)
+    T = 3
+    states = [O.CacheState() for _ in range(2)]
+    xs = x1s
+    for k in range(1, T + 1):
+        xs, _, _, sc = O.search_step(states, xs, k, T, 0.1, 1, 1, vel, target=y)
+    np.testing.assert_allclose(sc, [-np.linalg.norm(xs[i] - y) for i in range(2)], rtol=1e-15)
+
+
+# --------------------------------------------------------- search / select ---
+
+def test_topk_order_ties_and_nan():
+    assert O.topk([1.0, 3.0, 3.0, 2.0], 2).tolist() == [1, 2]
+    assert O.topk([np.nan, -5.0, 0.0], 3).tolist() == [2, 1, 0]
+    rng = np.random.default_rng(0)
+    for _ in range(50):
+        s = rng.integers(-3, 3, size=9).astype(float)
+        idx = O.topk(s, 9)
+        # brute force: descending by value, ascending index among equals
+        assert sorted(range(9), key=lambda i: (-s[i], i)) == idx.tolist()
+
+
+def test_cached_search_brute_force_argmax():
+    # Algorithm 1 on tiny inputs: argmax over independently scored rollouts
+    cfg, m = _tiny_model(blocks=1)
+    kv = m.text_kv(synth.text_context(cfg))
+    x1s = synth.initial_noise(cfg, range(4))
+    y = synth.target_latent(cfg)
+    vel = lambda x, t: m.velocity(x, t, kv)
+    i_star, scores, finals, _ = O.cached_search(x1s, 5, 0.1, 1, 1, vel, y)
+    brute = [-np.sqrt(((O.rollout(x1s[i], 5, 0.1, 1, 1, vel)[0] - y) ** 2).sum()) for i in range(4)]
+    np.testing.assert_allclose(scores, brute, rtol=1e-15)
+    assert scores[i_star] == max(scores)
+
+
+def test_beam_refill_layout_and_state_copy():
+    st = [O.CacheState(np.full(2, i * 1.0), np.full(2, 10.0 + i), 0.01 * i) for i in range(4)]
+    xs = np.arange(8, dtype=float).reshape(4, 2)
+    noise = np.ones((2 * 2, 2))
+    ns, nx = O.beam_refill(st, xs, [2, 0], 2, 0.1, noise)
+    assert len(ns) == 6
+    np.testing.assert_array_equal(nx[0], xs[2])
+    np.testing.assert_allclose(nx[1], xs[2] + 0.1)
+    np.testing.assert_array_equal(nx[3], xs[0])
+    assert ns[1].a == st[2].a and np.array_equal(ns[4].x_ref, st[0].x_ref)
+
+
+# --------------------------------------------------------------- primitives ---
+
+def test_attention_special_cases():
+    rng = np.random.default_rng(1)
+    v = rng.standard_normal((5, 4))
+    q = rng.standard_normal((3, 4))
+    # one key -> output is that value row
+    np.testing.assert_allclose(O.attention(q, rng.standard_normal((1, 4)), v[:1]), np.repeat(v[:1], 3, 0))
+    # identical keys -> uniform weights -> mean of V
+    k = np.repeat(rng.standard_normal((1, 4)), 5, 0)
+    np.testing.assert_allclose(O.attention(q, k, v), np.repeat(v.mean(0, keepdims=True), 3, 0), atol=1e-14)
+    # two keys with hand logits: q.k1/sqrt(4) = 0.5, q.k2 = 0 -> weights (s, 1-s), s = logistic(0.5)
+    s = 1 / (1 + math.exp(-0.5))
+    out = O.attention(np.ones((1, 4)), np.array([[1.0, 0, 0, 0], [0, 0, 0, 0]]), v[:2])
+    np.testing.assert_allclose(out[0], s * v[0] + (1 - s) * v[1], rtol=1e-13, atol=1e-15)
+
+
+def test_attention_rows_sum_to_one_and_match_torch_sdpa():
+    rng = np.random.default_rng(2)
+    q, k, v = (rng.standard_normal((37, 16)) for _ in range(3))
+    p = O.softmax_rows(q @ k.T / 4.0)
+    np.testing.assert_allclose(p.sum(1), 1.0, atol=1e-14)
+    ref = TF.scaled_dot_product_attention(*(torch.from_numpy(a)[None] for a in (q, k, v)))[0]
+    np.testing.assert_allclose(O.attention(q, k, v), ref.numpy(), atol=1e-12)
+
+
+def test_layer_norm_gelu_linear_against_independent_routines():
+    from scipy.special import erf
+    rng = np.random.default_rng(3)
+    x = rng.standard_normal((6, 10)) * 3 + 1
+    ref = TF.layer_norm(torch.from_numpy(x), (10,), eps=1e-6).numpy()
+    np.testing.assert_allclose(O.layer_norm(x), ref, atol=1e-12)
+    np.testing.assert_allclose(O.layer_norm(np.array([[-1.0, 1.0]])), [[-1 / math.sqrt(1 + 1e-6), 1 / math.sqrt(1 + 1e-6)]])
+    g = O.gelu_tanh(x)
+    np.testing.assert_allclose(g, TF.gelu(torch.from_numpy(x), approximate="tanh").numpy(), atol=1e-13)
+    # the tanh form stays within 1e-3 of the exact x Phi(x)
+    np.testing.assert_allclose(g, 0.5 * x * (1 + erf(x / math.sqrt(2))), atol=1e-3)
+    w = rng.standard_normal((3, 10))
+    b = rng.standard_normal(3)
+    np.testing.assert_allclose(O.linear(x, w, b), TF.linear(torch.from_numpy(x), torch.from_numpy(w), torch.from_numpy(b)).numpy(), atol=1e-12)
+    # non-square hand case: y = x W^T + b
+    np.testing.assert_allclose(O.linear(np.array([[1.0, 2.0]]), np.array([[1.0, 0.0], [0.0, 3.0], [1.0, 1.0]]), np.zeros(3)), [[1.0, 6.0, 3.0]])
+
+
+def test_patchify_layout_and_inverse():
+    C, F, H, W = 3, 2, 4, 6
+    x = np.arange(C * F * H * W, dtype=float).reshape(C, F, H, W)
+    tok = O.patchify(x)
+    assert tok.shape == (F * 2 * 3, C * 4)
+    for (c, f, h, w) in [(0, 0, 0, 0), (2, 1, 3, 5), (1, 0, 2, 1), (2, 1, 1, 4)]:
+        assert tok[(f * 2 + h // 2) * 3 + w // 2, c * 4 + (h % 2) * 2 + (w % 2)] == x[c, f, h, w]
+    np.testing.assert_array_equal(O.unpatchify(tok, C, F, H, W), x)
+
+
+def test_timestep_sinusoid_values():
+    e = O.timestep_sinusoid(0.0, 8)
+    np.testing.assert_array_equal(e, [1, 1, 1, 1, 0, 0, 0, 0])
+    e = O.timestep_sinusoid(0.5, 8)
+    # j = 0 has frequency 1: cos(500), sin(500); j = 2 has 10^-2: cos(5), sin(5)
+    np.testing.assert_allclose([e[0], e[4], e[2], e[6]], [math.cos(500), math.sin(500), math.cos(5), math.sin(5)], rtol=1e-12)
+
+
+def _block_torch(p, b, x, mod, kv, heads):
+    """The same block written with torch.nn.functional primitives (float64)."""
+    T = lambda a: torch.from_numpy(np.asarray(a, np.float64))
+    x = T(x)
+    d = x.shape[1]
+    hd = d // heads
+    sh1, sc1, g1, sh2, sc2, g2 = (T(m) for m in mod)
+    ln = lambda z: TF.layer_norm(z, (d,), eps=1e-6)
+
+    def mha(q, k, v):
+        sp = lambda z: z.reshape(z.shape[0], heads, hd).transpose(0, 1)
+        return TF.scaled_dot_product_attention(sp(q), sp(k), sp(v)).transpose(0, 1).reshape(q.shape[0], d)
+
+    h = ln(x) * (1 + sc1) + sh1
+    q, k, v = TF.linear(h, T(p[f"blk{b}.qkv_w"]), T(p[f"blk{b}.qkv_b"])).split(d, dim=1)
+    x = x + g1 * TF.linear(mha(q, k, v), T(p[f"blk{b}.o_w"]), T(p[f"blk{b}.o_b"]))
+    qc = TF.linear(ln(x), T(p[f"blk{b}.cq_w"]), T(p[f"blk{b}.cq_b"]))
+    x = x + TF.linear(mha(qc, T(kv[0]), T(kv[1])), T(p[f"blk{b}.co_w"]), T(p[f"blk{b}.co_b"]))
+    h = ln(x) * (1 + sc2) + sh2
+    f = TF.linear(TF.gelu(TF.linear(h, T(p[f"blk{b}.ff1_w"]), T(p[f"blk{b}.ff1_b"])), approximate="tanh"),
+                  T(p[f"blk{b}.ff2_w"]), T(p[f"blk{b}.ff2_b"]))
+    return (x + g2 * f).numpy()
+
+
+def test_block_against_torch_functional_composition():
+    cfg, m = _tiny_model(blocks=1)
+    rng = np.random.default_rng(4)
+    # random (non-zero) biases and offsets so that every term is exercised
+    for k in list(m.p):
+        if k.endswith("_b") or k.endswith("mod_off"):
+            m.p[k] = rng.standard_normal(m.p[k].shape) * 0.3
+    kv = m.text_kv(synth.text_context(cfg))
+    mods, _ = m.modulation(0.37)
+    x = rng.standard_normal((cfg.L, cfg.d))
+    np.testing.assert_allclose(m.block(0, x, mods[0], kv[0]),
+                               _block_torch(m.p, 0, x, mods[0], kv[0], cfg.heads), atol=1e-10)
+
+
+def test_dit_token_permutation_equivariance():
+    # no positional encoding: permuting video tokens permutes the velocity tokens
+    cfg, m = _tiny_model()
+    kv = m.text_kv(synth.text_context(cfg))
+    x = synth.initial_noise(cfg, [0])[0].astype(np.float64)
+    tok = O.patchify(x)
+    perm = np.random.default_rng(5).permutation(cfg.L)
+    v = O.patchify(m.velocity(x, 0.6, kv))
+    vp = O.patchify(m.velocity(O.unpatchify(tok[perm], cfg.C, cfg.F, cfg.H, cfg.W), 0.6, kv))
+    np.testing.assert_allclose(vp, v[perm], atol=1e-11)
+
+
+def test_dit_zero_blocks_reduce_to_head_of_embedding():
+    # all block weights 0 (and biases 0): every block is the identity, so
+    # v = head(LN(embed(x)) (1 + scale_h) + shift_h)
+    cfg, m = _tiny_model()
+    for k in list(m.p):
+        if k.startswith("blk"):
+            m.p[k] = np.zeros_like(m.p[k])
+    kv = m.text_kv(synth.text_context(cfg))
+    x = synth.initial_noise(cfg, [2])[0].astype(np.float64)
+    t = 0.25
+    _, hm = m.modulation(t)
+    tok = O.patchify(x) @ m.p["patch_w"].T
+    mu = tok.mean(1, keepdims=True)
+    sd = np.sqrt(tok.var(1, keepdims=True) + 1e-6)
+    out = ((tok - mu) / sd * (1 + hm[1]) + hm[0]) @ m.p["head_w"].T
+    np.testing.assert_allclose(O.patchify(m.velocity(x, t, kv)), out, atol=1e-12)
