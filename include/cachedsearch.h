@@ -1,0 +1,190 @@
+/*
+ * cachedsearch.h — C ABI of the GB300 (sm_103a) cached-search denoising step.
+ *
+ * Method: CachedSearch (arxiv 2607.23159).  N search candidates of a flow-matching
+ * video DiT are advanced one Euler step at a time (Sec. 2, Eq. euler).  For each
+ * candidate the adaptive transformation-vector cache (Sec. 3.1: Eq. delta, Eq. skip,
+ * Eq. indicator) decides whether the transformer runs; skipped candidates are
+ * compacted out of the transformer batch.  Candidates are scored and the best kept
+ * (Algorithm 1).
+ *
+ * Conventions shared by every call
+ *  - Pointers named *_dev are device pointers; ownership stays with the caller
+ *    unless stated.  Latent tensors are float32, candidate-major [N][D] with
+ *    D = C*F*H*W in (c, f, h, w) row-major order.
+ *  - Every call is asynchronous on the given stream unless it says it synchronises;
+ *    nothing is thrown across the ABI.  Each returns a cs_status; on failure
+ *    cs_last_error() gives a message for the calling thread.
+ *  - Kernels wait on nothing without a time limit: a wait that runs out records
+ *    CS_ERR_TIMEOUT in the device error word (read by cs_device_error()).
+ */
+#ifndef CACHEDSEARCH_H
+#define CACHEDSEARCH_H
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  CS_OK = 0,
+  CS_ERR_ARG = 1,         /* bad pointer, size or configuration                         */
+  CS_ERR_CUDA = 2,        /* a CUDA runtime/driver call failed (message has the reason)  */
+  CS_ERR_NONFINITE = 3,   /* a norm in the drift indicator was NaN/Inf or ||x_ref|| = 0   */
+  CS_ERR_TIMEOUT = 4,     /* a bounded device-side wait ran out                          */
+  CS_ERR_NOMEM = 5,       /* device allocation failed                                    */
+  CS_ERR_UNSUPPORTED = 6  /* shape outside what the kernels implement                    */
+} cs_status;
+
+/* Shape of the DiT velocity model v_theta(x, t, c) (Sec. 2) and of its latent. */
+typedef struct {
+  int C, F, H, W;   /* latent channels, frames, height, width (H, W even)               */
+  int d;            /* model width                                                      */
+  int heads;        /* attention heads; head dim d/heads must be 32 or 128              */
+  int ffn;          /* FFN hidden width                                                 */
+  int blocks;       /* transformer blocks                                               */
+  int f_dim;        /* timestep sinusoid features (even)                                */
+  int d_text;       /* raw text-embedding width                                         */
+  int Lt;           /* text tokens                                                      */
+  int max_batch;    /* most candidates one cs_search_step / cs_dit_forward call takes   */
+} cs_model_config;
+
+typedef struct cs_model cs_model;
+
+/* Message for the last failing call on this thread ("" if none). Never NULL. */
+const char* cs_last_error(void);
+
+/* Library version string. */
+const char* cs_version(void);
+
+/* Number of float32 parameters of a model of this shape (the length of the flat
+ * buffer cs_load_weights takes).  Layout, in order, Linear weights stored [out][in]
+ * (y = x W^T + b):
+ *   patch_w[d][4C] patch_b[d]  time_w1[d][f_dim] time_b1[d]  time_w2[d][d] time_b2[d]
+ *   mod_w[6d][d] mod_b[6d]  text_w1[d][d_text] text_b1[d]  text_w2[d][d] text_b2[d]
+ *   head_mod_w[2d][d] head_mod_b[2d]  head_w[4C][d] head_b[4C]
+ *   then per block: mod_off[6][d]  qkv_w[3d][d] qkv_b[3d]  o_w[d][d] o_b[d]
+ *   cq_w[d][d] cq_b[d]  ckv_w[2d][d] ckv_b[2d]  co_w[d][d] co_b[d]
+ *   ff1_w[ffn][d] ff1_b[ffn]  ff2_w[d][ffn] ff2_b[d]
+ * Returns 0 for an invalid configuration. */
+size_t cs_param_count(const cs_model_config* cfg);
+
+/* Create a model: validates the shape, allocates device weights and the workspace
+ * for cfg->max_batch candidates on the current device.  The library owns both;
+ * free them with cs_destroy_model.  Errors: CS_ERR_ARG (shape), CS_ERR_UNSUPPORTED,
+ * CS_ERR_NOMEM. */
+cs_status cs_init_model(const cs_model_config* cfg, cs_model** out);
+cs_status cs_destroy_model(cs_model* model);
+
+/* Load all parameters from a flat float32 buffer in the cs_param_count layout (host
+ * memory if params_on_device == 0, else device memory).  GEMM weights are stored as
+ * bf16 (round to nearest even), biases and the small conditioning MLPs as float32.
+ * Synchronises the stream. */
+cs_status cs_load_weights(cs_model* model, const float* params, size_t count, int params_on_device,
+                          cudaStream_t stream);
+
+/* Project the prompt's text context once per search: ctx_dev [Lt][d_text] float32
+ * (device).  Computes text = W2 GELU(W1 ctx + b1) + b2 and each block's
+ * cross-attention K/V, cached in the model for every later step (the prompt is shared
+ * by all candidates, Algorithm 1). */
+cs_status cs_set_text_context(cs_model* model, const float* ctx_dev, cudaStream_t stream);
+
+/* Velocity of a compacted subset: for j < n_c, v_dev[idx[j]] = v_theta(x_dev[idx[j]], t, c)
+ * (Sec. 2).  idx_dev: int32 [n_c] candidate indices (device); n_c <= max_batch.  Rows of
+ * v_dev not named in idx are left untouched. */
+cs_status cs_dit_forward(cs_model* model, const float* x_dev, const int32_t* idx_dev, int n_c, float t,
+                         float* v_dev, cudaStream_t stream);
+
+/* Bytes of scratch cs_cache_decide / cs_cache_apply / cs_score need for N candidates
+ * of D elements. */
+size_t cs_cache_workspace_bytes(int N, long long D);
+
+/* Cache rule, part 1 (Sec. 3.1, Eq. indicator).  For every candidate i at step k
+ * (1-based) of T:
+ *   forced_i = (k <= K_w) || (k > T - K_c) || !has_ref[i]
+ *   if !forced_i: a_i += ||x_i - x_ref_i||_F / ||x_ref_i||_F
+ *   compute_i = forced_i || tau <= 0 || a_i > tau     (tau <= 0 is "off": always compute)
+ *   force_compute (nullable, device u8 [N]) replaces compute_i after the accumulation.
+ *   computed candidates get a_i = 0 and has_ref_i = 1.
+ * Outputs: skip_mask_dev[i] = 1 if candidate i skips; compute_idx_dev [N] the indices
+ * of computing candidates in increasing order; n_compute_dev [1] their count.
+ * workspace_dev: cs_cache_workspace_bytes(N, D) bytes of device scratch.
+ * err_dev (nullable, device int): receives CS_ERR_NONFINITE when a norm is not finite
+ * or ||x_ref|| = 0 (that candidate is then computed), CS_ERR_ARG when force_compute
+ * asks an empty cache to skip. */
+cs_status cs_cache_decide(const float* x_dev, const float* x_ref_dev, float* accum_dev, uint8_t* has_ref_dev,
+                          int N, long long D, int step_k, int T, float tau, int K_w, int K_c,
+                          const uint8_t* force_compute_dev, uint8_t* skip_mask_dev, int32_t* compute_idx_dev,
+                          int32_t* n_compute_dev, void* workspace_dev, int* err_dev, cudaStream_t stream);
+
+/* Cache rule, part 2, fused with the Euler update (Eq. delta, Eq. skip, Eq. euler),
+ * h = t_next - t_cur:
+ *   skipped:  x += h (x + Delta)
+ *   computed: Delta = v - x;  x_ref = x;  x += h v       (v_dev [N][D], rows of computed candidates)
+ * If target_dev (device [D]) is given, scores_dev[i] = -||x0_i - target||_2 with the x0
+ * estimate x0_i = x_next_i - t_next * v_used_i (x_next itself on the last step). */
+cs_status cs_cache_apply(float* x_dev, float* x_ref_dev, float* delta_dev, const float* v_dev,
+                         const uint8_t* skip_mask_dev, int N, long long D, float t_cur, float t_next,
+                         const float* target_dev, float* scores_dev, void* workspace_dev, cudaStream_t stream);
+
+/* One denoising step of N candidates (the unit of work of the search):
+ * cs_cache_decide, then cs_dit_forward on the computing subset, then cs_cache_apply.
+ * State buffers (x, x_ref, delta: [N][D]; accum: [N]; has_ref: [N]) are caller-owned
+ * device memory and are updated in place; a fresh search starts with has_ref = 0.
+ * Synchronises once to read the number of computing candidates; that count is returned
+ * in *n_computed (host, nullable). */
+cs_status cs_search_step(cs_model* model, float* x_dev, float* x_ref_dev, float* delta_dev, float* accum_dev,
+                         uint8_t* has_ref_dev, int N, int step_k, int T, float t_cur, float t_next, float tau,
+                         int K_w, int K_c, const uint8_t* force_compute_dev, uint8_t* skip_mask_dev,
+                         const float* target_dev, float* scores_dev, int* n_computed, cudaStream_t stream);
+
+/* The same step with the latents in HOST memory (x_host [N][D], in/out) and the skip
+ * mask returned to HOST memory (skip_mask_host [N]); the cache state stays on the
+ * device.  Copies in, steps, copies out, and synchronises. */
+cs_status cs_search_step_host(cs_model* model, float* x_host, float* x_ref_dev, float* delta_dev,
+                              float* accum_dev, uint8_t* has_ref_dev, int N, int step_k, int T, float t_cur,
+                              float t_next, float tau, int K_w, int K_c, uint8_t* skip_mask_host,
+                              int* n_computed, cudaStream_t stream);
+
+/* scores_dev[i] = -||x_i - target||_2 (the verifier stand-in, Algorithm 1 "r_i <- V(y_i, c)"). */
+cs_status cs_score(const float* x_dev, const float* target_dev, int N, long long D, float* scores_dev,
+                   void* workspace_dev, cudaStream_t stream);
+
+/* Indices of the k largest scores in descending order (Algorithm 1, argmax when k = 1);
+ * equal scores keep the lower index first; NaN ranks below every number.  N <= 4096. */
+cs_status cs_select_topk(const float* scores_dev, int N, int k, int32_t* idx_dev, cudaStream_t stream);
+
+/* Beam refill: destination slot s = p*(1+children) + j takes the full state of
+ * candidate survivors[p] (x, x_ref, delta, accum, has_ref); for j > 0 (a child) it adds
+ * sigma * noise[p*children + j - 1] to x.  src and dst buffers must not overlap.
+ * survivors_dev: int32 [keep]; noise_dev: [keep*children][D]. */
+cs_status cs_beam_refill(const float* src_x, const float* src_x_ref, const float* src_delta,
+                         const float* src_accum, const uint8_t* src_has_ref, float* dst_x, float* dst_x_ref,
+                         float* dst_delta, float* dst_accum, uint8_t* dst_has_ref, const int32_t* survivors_dev,
+                         int keep, int children, float sigma, const float* noise_dev, long long D,
+                         cudaStream_t stream);
+
+/* First error recorded by the model's kernels since the last call (0 = none); clears
+ * it.  Synchronises the stream. */
+cs_status cs_device_error(cs_model* model, int* code, cudaStream_t stream);
+
+/* Per-kernel-class timing: when enabled, the model brackets every launch of the
+ * class with CUDA events on its stream.  Classes: 0 self-attention, 1 cross-attention,
+ * 2 GEMM, 3 cache decide+apply, 4 other.  cs_kernel_stats synchronises and returns
+ * the launches, summed milliseconds and algorithmic work (FLOPs for 0-2, bytes for 3)
+ * since the last reset. */
+cs_status cs_set_profiling(cs_model* model, int enable);
+cs_status cs_kernel_stats(cs_model* model, int kernel_class, long long* launches, double* total_ms,
+                          double* work);
+cs_status cs_reset_kernel_stats(cs_model* model);
+
+/* Kernel launches this library has issued in this process (all entry points). */
+long long cs_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* CACHEDSEARCH_H */

@@ -1,0 +1,358 @@
+// Flash attention forward on the tcgen05 tensor cores (self- and cross-attention of
+// the DiT blocks).  One CTA takes 256 query rows of one (batch item, head) as two
+// 128-row tiles A and B and streams the keys in tiles of 128:
+//
+//   warp 0      TMA producer: Q once, then K_j and V_j^T tiles through a 3-slot ring
+//   warp 1      TMEM allocator + MMA issuer, in the order
+//                 S_A(0) S_B(0) | PV_A(j) S_A(j+1) PV_B(j) S_B(j+1) | ...
+//               so that the tensor core works on one tile while the other's softmax runs
+//   warps 2..5  softmax of tile A, warps 6..9 softmax of tile B: one query row per
+//               thread; S row from TMEM, online max/sum in log2 units with lazy O
+//               rescaling (only when the running max grows by more than 8), P as bf16
+//               into shared memory in the 128-byte-swizzled K-major layout the MMA reads
+//
+// TMEM (512 columns): S_A [0,128), S_B [128,256), O_A [256, 256+hd), O_B [256+hd, 256+2hd).
+// S = Q K^T and O += P V are both M=128 tcgen05.mma with operands in shared memory;
+// V is stored transposed (V^T [hd][keys]) so that it is a K-major B operand.
+#include <cuda.h>
+#include <cuda_bf16.h>
+
+#include "common.cuh"
+#include "ptx.cuh"
+#include "tma_host.h"
+
+namespace cs {
+
+struct AttnArgs {
+  int B, heads, Lq, Lk, kv_shared;
+  float scale_log2;
+  __nv_bfloat16* o;
+  int* err;
+};
+
+template <int HD>
+struct AttnCfg {
+  static constexpr int HDS = HD < 64 ? 64 : HD;   // Q/K row length in shared memory
+  static constexpr int BQ = 128, BKV = 128;
+  static constexpr int QCH = HDS / 64;             // 64-wide chunks of a Q/K row
+  static constexpr int CH_BYTES = 128 * 64 * 2;    // one [128 x 64] bf16 chunk
+  static constexpr int Q_BYTES = QCH * CH_BYTES;   // one 128-row Q tile
+  static constexpr int K_BYTES = QCH * CH_BYTES;   // one 128-key K tile
+  static constexpr int VCH_BYTES = HD * 64 * 2;    // one [hd x 64 keys] chunk of V^T
+  static constexpr int V_BYTES = 2 * VCH_BYTES;
+  static constexpr int SLOT = K_BYTES > V_BYTES ? K_BYTES : V_BYTES;
+  static constexpr int NSLOT = 3;
+  static constexpr int P_BYTES = 2 * CH_BYTES;     // 128 rows x 128 keys
+  static constexpr int SMEM = 2 * Q_BYTES + NSLOT * SLOT + 2 * P_BYTES + 1024 + 256;
+  static constexpr uint32_t IDESC_S = idesc_bf16_f32(128, BKV);
+  static constexpr uint32_t IDESC_O = idesc_bf16_f32(128, HD);
+};
+
+template <int HD>
+__global__ void __launch_bounds__(320, 1)
+    attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                        const __grid_constant__ CUtensorMap tmV, const AttnArgs p) {
+  using Cfg = AttnCfg<HD>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = smem;                                   // [2][Q_BYTES]
+  uint8_t* sKV = sQ + 2 * Cfg::Q_BYTES;                 // [3][SLOT]
+  uint8_t* sP = sKV + Cfg::NSLOT * Cfg::SLOT;           // [2][P_BYTES]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + 2 * Cfg::P_BYTES);
+  uint64_t* q_full = bars;
+  uint64_t* kv_full = bars + 1;       // [3]
+  uint64_t* kv_empty = bars + 4;      // [3]
+  uint64_t* s_full = bars + 7;        // [2]
+  uint64_t* p_full = bars + 9;        // [2]
+  uint64_t* o_done = bars + 11;       // [2]
+  uint64_t* teardown = bars + 13;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 14);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int bh = blockIdx.y;
+  const int head = bh % p.heads, jb = bh / p.heads;
+  const int bkv = p.kv_shared ? head : bh;
+  const int q0 = blockIdx.x * 256;
+  const int nt = (p.Lk + Cfg::BKV - 1) / Cfg::BKV;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < 3; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+    }
+    for (int g = 0; g < 2; ++g) {
+      mbar_init(&s_full[g], 1);
+      mbar_init(&p_full[g], 128);
+      mbar_init(&o_done[g], 1);
+    }
+    mbar_init(teardown, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tmQ);
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      mbar_arrive_expect_tx(q_full, 2 * Cfg::Q_BYTES);
+      for (int g = 0; g < 2; ++g)
+        for (int c = 0; c < Cfg::QCH; ++c)
+          tma_load_3d(sQ + g * Cfg::Q_BYTES + c * Cfg::CH_BYTES, &tmQ, q_full, c * 64, q0 + g * 128, bh);
+      int issued = 0;
+      for (int s = 0; s < 2 * nt; ++s) {
+        const int slot = s % 3;
+        const uint32_t ph = (s / 3) & 1;
+        if (!mbar_wait(&kv_empty[slot], ph ^ 1, abort_flag, p.err)) break;
+        uint8_t* dst = sKV + slot * Cfg::SLOT;
+        const int j = s >> 1;
+        if ((s & 1) == 0) {
+          mbar_arrive_expect_tx(&kv_full[slot], Cfg::K_BYTES);
+          for (int c = 0; c < Cfg::QCH; ++c)
+            tma_load_3d(dst + c * Cfg::CH_BYTES, &tmK, &kv_full[slot], c * 64, j * Cfg::BKV, bkv);
+        } else {
+          mbar_arrive_expect_tx(&kv_full[slot], Cfg::V_BYTES);
+          for (int c = 0; c < 2; ++c)
+            tma_load_3d(dst + c * Cfg::VCH_BYTES, &tmV, &kv_full[slot], j * Cfg::BKV + c * 64, 0, bkv);
+        }
+        issued = s + 1;
+      }
+      if (*abort_flag) {
+        mbar_wait_teardown(q_full, 0);
+        for (int s = issued - 3 < 0 ? 0 : issued - 3; s < issued; ++s) mbar_wait_teardown(&kv_full[s % 3], (s / 3) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t tS[2] = {tmem_base, tmem_base + 128};
+      const uint32_t tO[2] = {tmem_base + 256, tmem_base + 256 + HD};
+      const uint32_t aQ[2] = {smem_u32(sQ), smem_u32(sQ + Cfg::Q_BYTES)};
+      const uint32_t aP[2] = {smem_u32(sP), smem_u32(sP + Cfg::P_BYTES)};
+      auto issue_s = [&](int g, uint32_t kslot) {
+#pragma unroll
+        for (int kk = 0; kk < Cfg::HDS / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * Cfg::CH_BYTES + (kk & 3) * 32;
+          umma_bf16_ss(tS[g], sdesc_sw128(aQ[g] + off), sdesc_sw128(kslot + off), Cfg::IDESC_S, kk > 0 ? 1u : 0u);
+        }
+        umma_commit(&s_full[g]);
+      };
+      auto issue_pv = [&](int g, uint32_t vslot, int j) {
+#pragma unroll
+        for (int kk = 0; kk < Cfg::BKV / 16; ++kk) {
+          const uint32_t offa = (kk >> 2) * Cfg::CH_BYTES + (kk & 3) * 32;
+          const uint32_t offb = (kk >> 2) * Cfg::VCH_BYTES + (kk & 3) * 32;
+          umma_bf16_ss(tO[g], sdesc_sw128(aP[g] + offa), sdesc_sw128(vslot + offb), Cfg::IDESC_O,
+                       (j > 0 || kk > 0) ? 1u : 0u);
+        }
+        umma_commit(&o_done[g]);
+      };
+      auto slot_addr = [&](int s) { return smem_u32(sKV + (s % 3) * Cfg::SLOT); };
+      bool ok = mbar_wait(q_full, 0, abort_flag, p.err);
+      if (ok) ok = mbar_wait(&kv_full[0], 0, abort_flag, p.err);
+      if (ok) {
+        tc_fence_after();
+        issue_s(0, slot_addr(0));
+        issue_s(1, slot_addr(0));
+        umma_commit(&kv_empty[0]);
+      }
+      for (int j = 0; ok && j < nt; ++j) {
+        const int sv = 2 * j + 1, sk = 2 * j + 2;
+        if (!mbar_wait(&kv_full[sv % 3], (sv / 3) & 1, abort_flag, p.err)) break;
+        if (!mbar_wait(&p_full[0], j & 1, abort_flag, p.err)) break;
+        tc_fence_after();
+        issue_pv(0, slot_addr(sv), j);
+        if (j + 1 < nt) {
+          if (!mbar_wait(&kv_full[sk % 3], (sk / 3) & 1, abort_flag, p.err)) break;
+          tc_fence_after();
+          issue_s(0, slot_addr(sk));
+        }
+        if (!mbar_wait(&p_full[1], j & 1, abort_flag, p.err)) break;
+        tc_fence_after();
+        issue_pv(1, slot_addr(sv), j);
+        umma_commit(&kv_empty[sv % 3]);
+        if (j + 1 < nt) {
+          issue_s(1, slot_addr(sk));
+          umma_commit(&kv_empty[sk % 3]);
+        }
+      }
+      if (*abort_flag) {
+        umma_commit(teardown);
+        mbar_wait_teardown(teardown, 0);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ softmax
+    const int g = (warp - 2) >> 2;          // 0: tile A (warps 2..5), 1: tile B (warps 6..9)
+    const int sp = warp & 3;                // TMEM lane quarter this warp may access
+    const int r = sp * 32 + lane;           // query row inside the tile
+    const uint32_t lane_off = (uint32_t)(sp * 32) << 16;
+    const uint32_t tS = tmem_base + lane_off + g * 128;
+    const uint32_t tO = tmem_base + lane_off + 256 + g * HD;
+    uint8_t* prow = sP + g * Cfg::P_BYTES + r * 128;
+    const float sl2 = p.scale_log2;
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nt; ++j) {
+      if (!mbar_wait(&s_full[g], j & 1, abort_flag, p.err)) { ok = false; break; }
+      tc_fence_after();
+      float x[128];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint32_t u[32];
+        tmem_ld32(tS + c * 32, u);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) x[c * 32 + e] = __uint_as_float(u[e]) * sl2;
+      }
+      const int valid = p.Lk - j * Cfg::BKV;
+      if (valid < Cfg::BKV) {
+#pragma unroll
+        for (int e = 0; e < 128; ++e)
+          if (e >= valid) x[e] = -INFINITY;
+      }
+      float mx = x[0];
+#pragma unroll
+      for (int e = 1; e < 128; ++e) mx = fmaxf(mx, x[e]);
+      const float m_new = fmaxf(m_run, mx);
+      const bool need = (j == 0) || (m_new > m_run + 8.f);
+      const bool warp_need = __any_sync(0xffffffffu, need);
+      const float m_use = need ? m_new : m_run;
+      const float factor = need ? ex2_approx(m_run - m_use) : 1.f;
+      float rs = 0.f;
+#pragma unroll
+      for (int e = 0; e < 128; ++e) {
+        x[e] = ex2_approx(x[e] - m_use);
+        rs += x[e];
+      }
+      l_run = l_run * factor + rs;
+      m_run = m_use;
+      if (j > 0) {
+        // PV of the previous tile must be done before O is rescaled and P overwritten
+        if (!mbar_wait(&o_done[g], (j - 1) & 1, abort_flag, p.err)) { ok = false; break; }
+        tc_fence_after();
+        if (warp_need) {
+#pragma unroll 1
+          for (int c = 0; c < HD / 32; ++c) {
+            uint32_t u[32];
+            tmem_ld32(tO + c * 32, u);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) u[e] = __float_as_uint(__uint_as_float(u[e]) * factor);
+            tmem_st32(tO + c * 32, u);
+          }
+        }
+      }
+      // P row -> shared memory, 128-byte swizzle: 16-byte unit u of row r sits at u ^ (r & 7)
+#pragma unroll
+      for (int cc = 0; cc < 2; ++cc) {
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const float* v = &x[cc * 64 + u * 8];
+          uint4 w;
+          w.x = pack_bf16x2(v[0], v[1]);
+          w.y = pack_bf16x2(v[2], v[3]);
+          w.z = pack_bf16x2(v[4], v[5]);
+          w.w = pack_bf16x2(v[6], v[7]);
+          *reinterpret_cast<uint4*>(prow + cc * Cfg::CH_BYTES + ((u ^ (r & 7)) << 4)) = w;
+        }
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(&p_full[g]);
+    }
+    if (ok && mbar_wait(&o_done[g], (nt - 1) & 1, abort_flag, p.err)) {
+      tc_fence_after();
+      const int q = q0 + g * 128 + r;
+      const float inv_l = 1.f / l_run;
+      const int d = p.heads * HD;
+      __nv_bfloat16* orow = p.o + ((long long)jb * p.Lq + q) * d + head * HD;
+#pragma unroll 1
+      for (int c = 0; c < HD / 32; ++c) {
+        uint32_t u[32];
+        tmem_ld32(tO + c * 32, u);
+        if (q < p.Lq) {
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+            uint4 o4;
+            o4.x = pack_bf16x2(__uint_as_float(u[8 * w + 0]) * inv_l, __uint_as_float(u[8 * w + 1]) * inv_l);
+            o4.y = pack_bf16x2(__uint_as_float(u[8 * w + 2]) * inv_l, __uint_as_float(u[8 * w + 3]) * inv_l);
+            o4.z = pack_bf16x2(__uint_as_float(u[8 * w + 4]) * inv_l, __uint_as_float(u[8 * w + 5]) * inv_l);
+            o4.w = pack_bf16x2(__uint_as_float(u[8 * w + 6]) * inv_l, __uint_as_float(u[8 * w + 7]) * inv_l);
+            reinterpret_cast<uint4*>(orow + c * 32)[w] = o4;
+          }
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, 512);
+  }
+}
+
+template <int HD>
+static cs_status launch_attn(const void* q, const void* k, const void* vt, void* o, int B, int heads, int Lq, int Lk,
+                             int Lkv_stride, int kv_shared, int* err, cudaStream_t stream) {
+  using Cfg = AttnCfg<HD>;
+  const int BH = B * heads, Bkv = kv_shared ? heads : BH;
+  CUtensorMap tq, tk, tv;
+  {
+    const uint64_t dims[3] = {(uint64_t)Cfg::HDS, (uint64_t)Lq, (uint64_t)BH};
+    const uint64_t str[2] = {(uint64_t)Cfg::HDS * 2, (uint64_t)Lq * Cfg::HDS * 2};
+    const uint32_t box[3] = {64, 128, 1};
+    CS_TRY(make_tmap_bf16(&tq, q, 3, dims, str, box));
+  }
+  {
+    const uint64_t dims[3] = {(uint64_t)Cfg::HDS, (uint64_t)Lk, (uint64_t)Bkv};
+    const uint64_t str[2] = {(uint64_t)Cfg::HDS * 2, (uint64_t)Lk * Cfg::HDS * 2};
+    const uint32_t box[3] = {64, 128, 1};
+    CS_TRY(make_tmap_bf16(&tk, k, 3, dims, str, box));
+  }
+  {
+    const uint64_t dims[3] = {(uint64_t)Lk, (uint64_t)HD, (uint64_t)Bkv};
+    const uint64_t str[2] = {(uint64_t)Lkv_stride * 2, (uint64_t)HD * Lkv_stride * 2};
+    const uint32_t box[3] = {64, (uint32_t)HD, 1};
+    CS_TRY(make_tmap_bf16(&tv, vt, 3, dims, str, box));
+  }
+  AttnArgs a{};
+  a.B = B; a.heads = heads; a.Lq = Lq; a.Lk = Lk; a.kv_shared = kv_shared;
+  a.scale_log2 = 1.4426950408889634f / sqrtf((float)HD);
+  a.o = static_cast<__nv_bfloat16*>(o);
+  a.err = err;
+  auto kern = attn_tcgen05_kernel<HD>;
+  CS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
+  dim3 grid((Lq + 255) / 256, BH);
+  kern<<<grid, 320, Cfg::SMEM, stream>>>(tq, tk, tv, a);
+  CS_LAUNCHED();
+  return CS_OK;
+}
+
+}  // namespace cs
+
+using namespace cs;
+
+extern "C" cs_status cs_attention(const void* q, const void* k, const void* vt, void* o, int B, int heads, int Lq,
+                                  int Lk, int hd, int Lkv_stride, int kv_shared, int* err, cudaStream_t stream) {
+  CS_REQUIRE(q && k && vt && o, "cs_attention: null pointer");
+  CS_REQUIRE(B > 0 && heads > 0 && Lq > 0 && Lk > 0, "cs_attention: empty shape");
+  CS_REQUIRE(Lkv_stride >= Lk && Lkv_stride % 8 == 0, "cs_attention: Lkv_stride must be >= Lk and a multiple of 8");
+  CS_REQUIRE((long long)B * heads <= 65535, "cs_attention: B*heads = %lld exceeds the grid limit",
+             (long long)B * heads);
+  if (hd == 128) return launch_attn<128>(q, k, vt, o, B, heads, Lq, Lk, Lkv_stride, kv_shared, err, stream);
+  if (hd == 32) return launch_attn<32>(q, k, vt, o, B, heads, Lq, Lk, Lkv_stride, kv_shared, err, stream);
+  set_error("cs_attention: head dim %d not supported (32 or 128)", hd);
+  return CS_ERR_UNSUPPORTED;
+}

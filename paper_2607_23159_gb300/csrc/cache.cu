@@ -1,0 +1,395 @@
+// Bandwidth-bound kernels of the cache rule, the Euler update, scoring and selection.
+//
+//  decide   Sec. 3.1 Eq. indicator: per-candidate ||x - x_ref||^2 and ||x_ref||^2 as
+//           fixed-order partial sums (128-bit loads, warp-shuffle trees), then one
+//           block turns them into a += drift, the skip decision and the compaction list.
+//  apply    Eq. delta / Eq. skip fused with Eq. euler (and, optionally, the x0-estimate
+//           score) in one pass over the candidate's latent.
+//  score    -||x - y*||_2 (the verifier stand-in of Algorithm 1).
+//  topk     rank-by-counting selection, deterministic tie-break.
+//  refill   beam refill (state copy of survivors + seeded perturbation of children).
+//
+// Every reduction's order depends only on D (never on N or on which candidates are
+// present), so a candidate's numbers are the same whatever batch it is in.
+#include <cmath>
+#include <cstdint>
+
+#include "common.cuh"
+#include "ptx.cuh"
+
+namespace cs {
+
+constexpr int kCacheThreads = 256;
+constexpr long long kChunkElems = 32768;   // elements of one candidate per CTA (multiple of 4*256)
+
+__host__ __device__ inline int cache_chunks(long long D) {
+  long long c = (D + kChunkElems - 1) / kChunkElems;
+  return (int)(c < 1 ? 1 : c);
+}
+
+// Block-wide sum of two values in a fixed order (warp shuffle tree, then warp 0).
+template <int NV>
+__device__ __forceinline__ void block_sum(float (&v)[NV], float (*red)[32]) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int q = 0; q < NV; ++q) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v[q] += __shfl_xor_sync(0xffffffffu, v[q], o);
+  }
+  if (lane == 0) {
+#pragma unroll
+    for (int q = 0; q < NV; ++q) red[q][warp] = v[q];
+  }
+  __syncthreads();
+  if (warp == 0) {
+    const int nw = blockDim.x >> 5;
+#pragma unroll
+    for (int q = 0; q < NV; ++q) {
+      float s = lane < nw ? red[q][lane] : 0.f;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+      v[q] = s;
+    }
+  }
+}
+
+__host__ __device__ __forceinline__ bool window_forced(int k, int T, int K_w, int K_c) {
+  return k <= K_w || k > T - K_c;
+}
+
+// ------------------------------------------------------------------ decide ----
+__global__ void __launch_bounds__(kCacheThreads) drift_partials_kernel(
+    const float* __restrict__ x, const float* __restrict__ xr, const uint8_t* __restrict__ has_ref, long long D,
+    int window_forced_step, float* __restrict__ partials) {
+  const int i = blockIdx.y, c = blockIdx.x, nch = gridDim.x;
+  __shared__ float red[2][32];
+  if (window_forced_step || !has_ref[i]) return;   // forced step: no drift is evaluated
+  const long long lo = (long long)c * kChunkElems;
+  const long long hi = min(D, lo + kChunkElems);
+  const float* xi = x + (long long)i * D;
+  const float* ri = xr + (long long)i * D;
+  float v[2] = {0.f, 0.f};
+  const bool vec = ((D & 3) == 0) && ((reinterpret_cast<uintptr_t>(x) & 15) == 0) &&
+                   ((reinterpret_cast<uintptr_t>(xr) & 15) == 0);
+  if (vec) {
+    const float4* x4 = reinterpret_cast<const float4*>(xi + lo);
+    const float4* r4 = reinterpret_cast<const float4*>(ri + lo);
+    const int n4 = (int)((hi - lo) >> 2);
+#pragma unroll 4
+    for (int e = threadIdx.x; e < n4; e += kCacheThreads) {
+      const float4 a = __ldcs(x4 + e), b = __ldcs(r4 + e);
+      const float d0 = a.x - b.x, d1 = a.y - b.y, d2 = a.z - b.z, d3 = a.w - b.w;
+      v[0] += d0 * d0 + d1 * d1 + d2 * d2 + d3 * d3;
+      v[1] += b.x * b.x + b.y * b.y + b.z * b.z + b.w * b.w;
+    }
+  } else {
+    for (long long e = lo + threadIdx.x; e < hi; e += kCacheThreads) {
+      const float a = xi[e], b = ri[e];
+      v[0] += (a - b) * (a - b);
+      v[1] += b * b;
+    }
+  }
+  block_sum<2>(v, red);
+  if (threadIdx.x == 0) {
+    partials[((long long)i * nch + c) * 2 + 0] = v[0];
+    partials[((long long)i * nch + c) * 2 + 1] = v[1];
+  }
+}
+
+__global__ void decide_finalize_kernel(const float* __restrict__ partials, int nch, float* __restrict__ accum,
+                                       uint8_t* __restrict__ has_ref, int N, int window_forced_step, float tau,
+                                       const uint8_t* __restrict__ force, uint8_t* __restrict__ skip_mask,
+                                       int32_t* __restrict__ idx, int32_t* __restrict__ n_compute, int* err) {
+  extern __shared__ uint8_t flags[];
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    const bool had = has_ref[i] != 0;
+    bool compute;
+    float a = accum[i];
+    if (window_forced_step || !had) {
+      compute = true;
+    } else {
+      double num = 0.0, den = 0.0;
+      for (int c = 0; c < nch; ++c) {
+        num += (double)partials[((long long)i * nch + c) * 2 + 0];
+        den += (double)partials[((long long)i * nch + c) * 2 + 1];
+      }
+      const double drift = sqrt(num) / sqrt(den);
+      if (!isfinite(drift)) {
+        record_error(err, CS_ERR_NONFINITE);
+        compute = true;
+      } else {
+        a = (float)((double)a + drift);
+        compute = (tau <= 0.f) || (a > tau);
+      }
+    }
+    if (force) {
+      const bool f = force[i] != 0;
+      if (!f && !had) {
+        record_error(err, CS_ERR_ARG);
+      } else {
+        compute = f;
+      }
+    }
+    if (compute) {
+      a = 0.f;
+      has_ref[i] = 1;
+    }
+    accum[i] = a;
+    skip_mask[i] = compute ? 0 : 1;
+    flags[i] = compute ? 1 : 0;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int n = 0;
+    for (int i = 0; i < N; ++i)
+      if (flags[i]) idx[n++] = i;
+    *n_compute = n;
+  }
+}
+
+// ------------------------------------------------------------------- apply ----
+template <bool kScore>
+__global__ void __launch_bounds__(kCacheThreads) apply_kernel(float* __restrict__ x, float* __restrict__ xr,
+                                                              float* __restrict__ delta,
+                                                              const float* __restrict__ v,
+                                                              const uint8_t* __restrict__ skip, long long D,
+                                                              float h, float t_next,
+                                                              const float* __restrict__ target,
+                                                              float* __restrict__ partials) {
+  const int i = blockIdx.y, c = blockIdx.x, nch = gridDim.x;
+  __shared__ float red[1][32];
+  const long long lo = (long long)c * kChunkElems;
+  const long long hi = min(D, lo + kChunkElems);
+  const long long base = (long long)i * D;
+  const bool skipped = skip[i] != 0;
+  float acc[1] = {0.f};
+  const bool vec = ((D & 3) == 0) && ((reinterpret_cast<uintptr_t>(x) & 15) == 0) &&
+                   ((reinterpret_cast<uintptr_t>(xr) & 15) == 0) &&
+                   ((reinterpret_cast<uintptr_t>(delta) & 15) == 0) &&
+                   ((reinterpret_cast<uintptr_t>(v) & 15) == 0) &&
+                   (!kScore || (reinterpret_cast<uintptr_t>(target) & 15) == 0);
+  if (vec) {
+    float4* x4 = reinterpret_cast<float4*>(x + base + lo);
+    float4* r4 = reinterpret_cast<float4*>(xr + base + lo);
+    float4* d4 = reinterpret_cast<float4*>(delta + base + lo);
+    const float4* v4 = reinterpret_cast<const float4*>(v + base + lo);
+    const float4* y4 = reinterpret_cast<const float4*>(target + lo);
+    const int n4 = (int)((hi - lo) >> 2);
+#pragma unroll 2
+    for (int e = threadIdx.x; e < n4; e += kCacheThreads) {
+      const float4 xv = __ldcs(x4 + e);
+      float4 vu, xn;
+      if (skipped) {   // Eq. skip: v_hat = x + Delta
+        const float4 dv = __ldcs(d4 + e);
+        vu = make_float4(xv.x + dv.x, xv.y + dv.y, xv.z + dv.z, xv.w + dv.w);
+      } else {         // Eq. delta: Delta = v - x, x_ref = x
+        vu = __ldcs(v4 + e);
+        __stcs(d4 + e, make_float4(vu.x - xv.x, vu.y - xv.y, vu.z - xv.z, vu.w - xv.w));
+        __stcs(r4 + e, xv);
+      }
+      xn = make_float4(xv.x + h * vu.x, xv.y + h * vu.y, xv.z + h * vu.z, xv.w + h * vu.w);   // Eq. euler
+      __stcs(x4 + e, xn);
+      if (kScore) {
+        const float4 y = __ldg(y4 + e);
+        const float e0 = xn.x - t_next * vu.x - y.x, e1 = xn.y - t_next * vu.y - y.y;
+        const float e2 = xn.z - t_next * vu.z - y.z, e3 = xn.w - t_next * vu.w - y.w;
+        acc[0] += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
+      }
+    }
+  } else {
+    for (long long e = lo + threadIdx.x; e < hi; e += kCacheThreads) {
+      const float xv = x[base + e];
+      float vu;
+      if (skipped) {
+        vu = xv + delta[base + e];
+      } else {
+        vu = v[base + e];
+        delta[base + e] = vu - xv;
+        xr[base + e] = xv;
+      }
+      const float xn = xv + h * vu;
+      x[base + e] = xn;
+      if (kScore) {
+        const float d0 = xn - t_next * vu - target[e];
+        acc[0] += d0 * d0;
+      }
+    }
+  }
+  if (kScore) {
+    block_sum<1>(acc, red);
+    if (threadIdx.x == 0) partials[(long long)i * nch + c] = acc[0];
+  }
+}
+
+// ------------------------------------------------------------------- score ----
+__global__ void __launch_bounds__(kCacheThreads) sqdist_partials_kernel(const float* __restrict__ x,
+                                                                        const float* __restrict__ y, long long D,
+                                                                        float* __restrict__ partials) {
+  const int i = blockIdx.y, c = blockIdx.x, nch = gridDim.x;
+  __shared__ float red[1][32];
+  const long long lo = (long long)c * kChunkElems;
+  const long long hi = min(D, lo + kChunkElems);
+  const float* xi = x + (long long)i * D;
+  float acc[1] = {0.f};
+  const bool vec = ((D & 3) == 0) && ((reinterpret_cast<uintptr_t>(x) & 15) == 0) &&
+                   ((reinterpret_cast<uintptr_t>(y) & 15) == 0);
+  if (vec) {
+    const float4* x4 = reinterpret_cast<const float4*>(xi + lo);
+    const float4* y4 = reinterpret_cast<const float4*>(y + lo);
+    const int n4 = (int)((hi - lo) >> 2);
+    for (int e = threadIdx.x; e < n4; e += kCacheThreads) {
+      const float4 a = __ldcs(x4 + e), b = __ldg(y4 + e);
+      const float d0 = a.x - b.x, d1 = a.y - b.y, d2 = a.z - b.z, d3 = a.w - b.w;
+      acc[0] += d0 * d0 + d1 * d1 + d2 * d2 + d3 * d3;
+    }
+  } else {
+    for (long long e = lo + threadIdx.x; e < hi; e += kCacheThreads) {
+      const float d0 = xi[e] - y[e];
+      acc[0] += d0 * d0;
+    }
+  }
+  block_sum<1>(acc, red);
+  if (threadIdx.x == 0) partials[(long long)i * nch + c] = acc[0];
+}
+
+__global__ void score_finalize_kernel(const float* __restrict__ partials, int nch, int N,
+                                      float* __restrict__ scores) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < N; i += gridDim.x * blockDim.x) {
+    double s = 0.0;
+    for (int c = 0; c < nch; ++c) s += (double)partials[(long long)i * nch + c];
+    scores[i] = (float)(-sqrt(s));
+  }
+}
+
+// -------------------------------------------------------------------- top-k ----
+__global__ void topk_kernel(const float* __restrict__ scores, int N, int k, int32_t* __restrict__ idx) {
+  extern __shared__ float s[];
+  for (int i = threadIdx.x; i < N; i += blockDim.x) s[i] = scores[i];
+  __syncthreads();
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    const float si = s[i];
+    const bool ni = isnan(si);
+    int rank = 0;
+    for (int j = 0; j < N; ++j) {
+      const float sj = s[j];
+      const bool nj = isnan(sj);
+      const bool greater = (!nj && ni) || (!nj && !ni && sj > si);
+      const bool equal = (nj && ni) || (!nj && !ni && sj == si);
+      rank += (greater || (equal && j < i)) ? 1 : 0;
+    }
+    if (rank < k) idx[rank] = i;
+  }
+}
+
+// ------------------------------------------------------------------ refill ----
+__global__ void __launch_bounds__(kCacheThreads) beam_refill_kernel(
+    const float* __restrict__ sx, const float* __restrict__ sr, const float* __restrict__ sd,
+    const float* __restrict__ sa, const uint8_t* __restrict__ sh, float* __restrict__ dx, float* __restrict__ dr,
+    float* __restrict__ dd, float* __restrict__ da, uint8_t* __restrict__ dh, const int32_t* __restrict__ surv,
+    int children, float sigma, const float* __restrict__ noise, long long D) {
+  const int slot = blockIdx.y, c = blockIdx.x;
+  const int p = slot / (children + 1), j = slot % (children + 1);
+  const int src = surv[p];
+  const long long lo = (long long)c * kChunkElems;
+  const long long hi = min(D, lo + kChunkElems);
+  const long long so = (long long)src * D, dof = (long long)slot * D;
+  const float* nz = j > 0 ? noise + (long long)(p * children + j - 1) * D : nullptr;
+  for (long long e = lo + threadIdx.x; e < hi; e += kCacheThreads) {
+    float xv = sx[so + e];
+    if (nz) xv += sigma * nz[e];
+    dx[dof + e] = xv;
+    dr[dof + e] = sr[so + e];
+    dd[dof + e] = sd[so + e];
+  }
+  if (c == 0 && threadIdx.x == 0) {
+    da[slot] = sa[src];
+    dh[slot] = sh[src];
+  }
+}
+
+}  // namespace cs
+
+using namespace cs;
+
+extern "C" size_t cs_cache_workspace_bytes(int N, long long D) {
+  if (N <= 0 || D <= 0) return 0;
+  return (size_t)N * (size_t)cache_chunks(D) * 3 * sizeof(float);
+}
+
+extern "C" cs_status cs_cache_decide(const float* x, const float* x_ref, float* accum, uint8_t* has_ref, int N,
+                                     long long D, int step_k, int T, float tau, int K_w, int K_c,
+                                     const uint8_t* force, uint8_t* skip_mask, int32_t* idx, int32_t* n_compute,
+                                     void* workspace, int* err, cudaStream_t stream) {
+  CS_REQUIRE(N > 0 && N <= 4096 && D > 0, "cs_cache_decide: need 0 < N <= 4096 and D > 0 (N=%d D=%lld)", N, D);
+  CS_REQUIRE(x && x_ref && accum && has_ref && skip_mask && idx && n_compute && workspace,
+             "cs_cache_decide: null pointer");
+  CS_REQUIRE(step_k >= 1 && step_k <= T, "cs_cache_decide: step %d outside 1..T=%d", step_k, T);
+  const int nch = cache_chunks(D);
+  const int wf = window_forced(step_k, T, K_w, K_c) ? 1 : 0;
+  float* partials = static_cast<float*>(workspace);
+  if (!wf) {
+    drift_partials_kernel<<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, has_ref, D, wf, partials);
+    CS_LAUNCHED();
+  }
+  decide_finalize_kernel<<<1, 256, N, stream>>>(partials, nch, accum, has_ref, N, wf, tau, force, skip_mask, idx,
+                                                n_compute, err);
+  CS_LAUNCHED();
+  return CS_OK;
+}
+
+extern "C" cs_status cs_cache_apply(float* x, float* x_ref, float* delta, const float* v, const uint8_t* skip_mask,
+                                    int N, long long D, float t_cur, float t_next, const float* target,
+                                    float* scores, void* workspace, cudaStream_t stream) {
+  CS_REQUIRE(N > 0 && N <= 4096 && D > 0, "cs_cache_apply: need 0 < N <= 4096 and D > 0");
+  CS_REQUIRE(x && x_ref && delta && v && skip_mask, "cs_cache_apply: null pointer");
+  CS_REQUIRE(!target || (scores && workspace), "cs_cache_apply: scoring needs scores and workspace");
+  const int nch = cache_chunks(D);
+  const float h = t_next - t_cur;
+  float* partials = workspace ? static_cast<float*>(workspace) + (size_t)N * nch * 2 : nullptr;
+  if (target) {
+    apply_kernel<true><<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, delta, v, skip_mask, D, h, t_next,
+                                                                   target, partials);
+    CS_LAUNCHED();
+    score_finalize_kernel<<<(N + 127) / 128, 128, 0, stream>>>(partials, nch, N, scores);
+    CS_LAUNCHED();
+  } else {
+    apply_kernel<false><<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, delta, v, skip_mask, D, h, t_next,
+                                                                    nullptr, nullptr);
+    CS_LAUNCHED();
+  }
+  return CS_OK;
+}
+
+extern "C" cs_status cs_score(const float* x, const float* target, int N, long long D, float* scores,
+                              void* workspace, cudaStream_t stream) {
+  CS_REQUIRE(N > 0 && N <= 4096 && D > 0 && x && target && scores && workspace, "cs_score: bad arguments");
+  const int nch = cache_chunks(D);
+  float* partials = static_cast<float*>(workspace) + (size_t)N * nch * 2;
+  sqdist_partials_kernel<<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, target, D, partials);
+  CS_LAUNCHED();
+  score_finalize_kernel<<<(N + 127) / 128, 128, 0, stream>>>(partials, nch, N, scores);
+  CS_LAUNCHED();
+  return CS_OK;
+}
+
+extern "C" cs_status cs_select_topk(const float* scores, int N, int k, int32_t* idx, cudaStream_t stream) {
+  CS_REQUIRE(N > 0 && N <= 4096 && k >= 1 && k <= N && scores && idx, "cs_select_topk: need 1 <= k <= N <= 4096");
+  topk_kernel<<<1, 256, N * sizeof(float), stream>>>(scores, N, k, idx);
+  CS_LAUNCHED();
+  return CS_OK;
+}
+
+extern "C" cs_status cs_beam_refill(const float* sx, const float* sr, const float* sd, const float* sa,
+                                    const uint8_t* sh, float* dx, float* dr, float* dd, float* da, uint8_t* dh,
+                                    const int32_t* surv, int keep, int children, float sigma, const float* noise,
+                                    long long D, cudaStream_t stream) {
+  CS_REQUIRE(keep > 0 && children >= 0 && D > 0, "cs_beam_refill: bad sizes");
+  CS_REQUIRE(sx && sr && sd && sa && sh && dx && dr && dd && da && dh && surv && (children == 0 || noise),
+             "cs_beam_refill: null pointer");
+  CS_REQUIRE(sx != dx && sr != dr && sd != dd, "cs_beam_refill: source and destination must differ");
+  const int slots = keep * (children + 1);
+  beam_refill_kernel<<<dim3(cache_chunks(D), slots), kCacheThreads, 0, stream>>>(
+      sx, sr, sd, sa, sh, dx, dr, dd, da, dh, surv, children, sigma, noise, D);
+  CS_LAUNCHED();
+  return CS_OK;
+}

@@ -1,0 +1,30 @@
+// Internal interfaces between the library's translation units.
+#pragma once
+#include <cstdint>
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "../../include/cachedsearch.h"
+
+namespace cs {
+
+struct CondWeights {
+  int d, f_dim, blocks;
+  const __nv_bfloat16 *time_w1, *time_w2, *mod_w, *head_mod_w;
+  const float *time_b1, *time_b2, *mod_b, *head_mod_b;
+  const float* const* mod_offs;   // device array of `blocks` pointers to [6][d]
+};
+
+// scratch: f_dim + 9 d floats; mods: [blocks][6][d]; hmod: [2][d] (shift, scale)
+cs_status timestep_conditioning(const CondWeights& w, float t, float* scratch, float* mods, float* hmod,
+                                cudaStream_t s);
+cs_status layernorm_modulate(const float* x, const float* shift, const float* scale, __nv_bfloat16* out, int M, int d,
+                             cudaStream_t s);
+cs_status patchify(const float* x, const int32_t* idx, int n_c, int C, int F, int H, int W, int Kp,
+                   __nv_bfloat16* tok, cudaStream_t s);
+cs_status unpatchify(const float* hout, const int32_t* idx, int n_c, int C, int F, int H, int W, float* v,
+                     cudaStream_t s);
+cs_status to_bf16_pad(const float* src, long long rows, int cols, int ld, __nv_bfloat16* dst, cudaStream_t s);
+
+}  // namespace cs

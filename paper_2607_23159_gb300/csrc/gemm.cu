@@ -1,0 +1,362 @@
+// tcgen05 GEMM for the DiT's Linear layers: C = A B^T, bf16 operands staged by TMA
+// (128-byte swizzle) in a shared-memory ring, float32 accumulators in TMEM, fused
+// epilogues (bias, GELU, gated residual add, attention-layout scatter).
+//
+// Persistent kernel, one CTA per SM, 6 warps:
+//   warp 0      TMA producer (one lane): A tile 128 x 64 and B tile BN x 64 per stage
+//   warp 1      TMEM allocator + MMA issuer (one lane): 4 x tcgen05.mma (K = 16) per stage
+//   warps 2..5  epilogue: tcgen05.ld of the 128 x BN accumulator (warp w reads TMEM
+//               lanes 32*(w%4)..+31), bias/activation, global stores
+// Two TMEM accumulators (2 x BN columns) let the epilogue of tile i overlap the main
+// loop of tile i+1.  Tiles are visited n-fastest so that the CTAs in flight share A
+// rows and the whole of B in L2.
+#include <cuda.h>
+#include <cuda_bf16.h>
+
+#include "common.cuh"
+#include "ptx.cuh"
+#include "tma_host.h"
+
+namespace cs {
+
+struct GemmArgs {
+  int M, N, K;
+  const float* bias;
+  const float* gate;
+  void* out;
+  int ldo;
+  // attention-layout scatter (CS_EPI_QKV)
+  __nv_bfloat16* q;
+  __nv_bfloat16* k;
+  __nv_bfloat16* vt;
+  int L, d, heads, hd, hd_s, Lv, which_base;
+  int* err;
+};
+
+template <int BN>
+struct GemmCfg {
+  static constexpr int BM = 128, BK = 64;
+  static constexpr int STAGES = BN == 256 ? 4 : 6;
+  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int TMEM_COLS = 2 * BN;
+  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+  static constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
+};
+
+__device__ __forceinline__ float gelu_tanh(float x) {
+  // 0.5 x (1 + tanh(sqrt(2/pi) (x + 0.044715 x^3)))  (Hendrycks & Gimpel 2016)
+  const float k0 = 0.7978845608028654f, k1 = 0.044715f;
+  return 0.5f * x * (1.f + tanhf(k0 * (x + k1 * x * x * x)));
+}
+
+// One thread's 32 consecutive accumulator columns [n, n+32) of row m.
+template <int EPI>
+__device__ __forceinline__ void epilogue_chunk(const GemmArgs& p, int m, int n, const uint32_t (&r)[32]) {
+  float f[32];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) f[j] = __uint_as_float(r[j]);
+  const bool full = (n + 32 <= p.N);
+  if (p.bias) {
+    if (full) {
+      const float4* b4 = reinterpret_cast<const float4*>(p.bias + n);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float4 b = __ldg(b4 + j);
+        f[4 * j] += b.x; f[4 * j + 1] += b.y; f[4 * j + 2] += b.z; f[4 * j + 3] += b.w;
+      }
+    } else {
+      for (int j = 0; j < 32; ++j)
+        if (n + j < p.N) f[j] += __ldg(p.bias + n + j);
+    }
+  }
+  if constexpr (EPI == CS_EPI_F32) {
+    float* o = static_cast<float*>(p.out) + (long long)m * p.ldo + n;
+    if (full && (p.ldo % 4) == 0) {
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        reinterpret_cast<float4*>(o)[j] = make_float4(f[4 * j], f[4 * j + 1], f[4 * j + 2], f[4 * j + 3]);
+    } else {
+      for (int j = 0; j < 32; ++j)
+        if (n + j < p.N) o[j] = f[j];
+    }
+  } else if constexpr (EPI == CS_EPI_BF16 || EPI == CS_EPI_GELU_BF16) {
+    if constexpr (EPI == CS_EPI_GELU_BF16) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) f[j] = gelu_tanh(f[j]);
+    }
+    __nv_bfloat16* o = static_cast<__nv_bfloat16*>(p.out) + (long long)m * p.ldo + n;
+    if (full && (p.ldo % 8) == 0) {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        uint4 u;
+        u.x = pack_bf16x2(f[8 * j + 0], f[8 * j + 1]);
+        u.y = pack_bf16x2(f[8 * j + 2], f[8 * j + 3]);
+        u.z = pack_bf16x2(f[8 * j + 4], f[8 * j + 5]);
+        u.w = pack_bf16x2(f[8 * j + 6], f[8 * j + 7]);
+        reinterpret_cast<uint4*>(o)[j] = u;
+      }
+    } else {
+      for (int j = 0; j < 32; ++j)
+        if (n + j < p.N) o[j] = __float2bfloat16_rn(f[j]);
+    }
+  } else if constexpr (EPI == CS_EPI_RESID_F32) {
+    float* o = static_cast<float*>(p.out) + (long long)m * p.ldo + n;
+    if (full && (p.ldo % 4) == 0) {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        float4 x = reinterpret_cast<float4*>(o)[j];
+        float4 g = p.gate ? __ldg(reinterpret_cast<const float4*>(p.gate + n) + j) : make_float4(1.f, 1.f, 1.f, 1.f);
+        x.x += g.x * f[4 * j]; x.y += g.y * f[4 * j + 1]; x.z += g.z * f[4 * j + 2]; x.w += g.w * f[4 * j + 3];
+        reinterpret_cast<float4*>(o)[j] = x;
+      }
+    } else {
+      for (int j = 0; j < 32; ++j)
+        if (n + j < p.N) o[j] += (p.gate ? __ldg(p.gate + n + j) : 1.f) * f[j];
+    }
+  } else if constexpr (EPI == CS_EPI_QKV) {
+    // 32 | hd, so the chunk lies inside one head of one projection
+    const int w = p.which_base + n / p.d;
+    const int c0 = n % p.d;
+    const int head = c0 / p.hd, e = c0 % p.hd;
+    const int jb = m / p.L, l = m % p.L;
+    const long long bh = (long long)jb * p.heads + head;
+    if (w < 2) {
+      __nv_bfloat16* o = (w == 0 ? p.q : p.k) + (bh * p.L + l) * p.hd_s + e;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        uint4 u;
+        u.x = pack_bf16x2(f[8 * j + 0], f[8 * j + 1]);
+        u.y = pack_bf16x2(f[8 * j + 2], f[8 * j + 3]);
+        u.z = pack_bf16x2(f[8 * j + 4], f[8 * j + 5]);
+        u.w = pack_bf16x2(f[8 * j + 6], f[8 * j + 7]);
+        reinterpret_cast<uint4*>(o)[j] = u;
+      }
+    } else {
+      __nv_bfloat16* o = p.vt + (bh * p.hd + e) * p.Lv + l;
+#pragma unroll
+      for (int j = 0; j < 32; ++j) o[(long long)j * p.Lv] = __float2bfloat16_rn(f[j]);
+    }
+  }
+}
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(192, 1)
+    gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                        const GemmArgs p) {
+  using Cfg = GemmCfg<BN>;
+  constexpr int BM = Cfg::BM, BK = Cfg::BK, STAGES = Cfg::STAGES;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * Cfg::A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * Cfg::STAGE_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* tfull = empty + STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* teardown = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(teardown + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 4);
+    }
+    mbar_init(teardown, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int m_tiles = (p.M + BM - 1) / BM, n_tiles = (p.N + BN - 1) / BN;
+  const int tiles = m_tiles * n_tiles;
+  const int kblocks = p.K / BK;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tma_prefetch_desc(&tmA);
+      tma_prefetch_desc(&tmB);
+      int stage = 0;
+      uint32_t phase = 0;
+      int issued = 0;
+      for (int tile = blockIdx.x; tile < tiles && !*abort_flag; tile += gridDim.x) {
+        const int m0 = (tile / n_tiles) * BM, n0 = (tile % n_tiles) * BN;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.err)) break;
+          mbar_arrive_expect_tx(&full[stage], Cfg::STAGE_BYTES);
+          tma_load_2d(sA + stage * Cfg::A_BYTES, &tmA, &full[stage], kb * BK, m0);
+          tma_load_2d(sB + stage * Cfg::B_BYTES, &tmB, &full[stage], kb * BK, n0);
+          ++issued;
+          if (++stage == STAGES) { stage = 0; phase ^= 1; }
+        }
+      }
+      if (*abort_flag) {
+        // drain: wait (bounded) for the loads of the last ring's worth of stages
+        for (int back = 1; back <= STAGES && back <= issued; ++back) {
+          int s = stage - back, ph = phase;
+          if (s < 0) { s += STAGES; ph ^= 1; }
+          mbar_wait_teardown(&full[s], ph);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      for (int tile = blockIdx.x; tile < tiles && !*abort_flag; tile += gridDim.x) {
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.err)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        bool ok = true;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag, p.err)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + stage * Cfg::A_BYTES);
+          const uint32_t b0 = smem_u32(sB + stage * Cfg::B_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            umma_bf16_ss(d_tmem, sdesc_sw128(a0 + k * 32), sdesc_sw128(b0 + k * 32), Cfg::IDESC,
+                         (kb | k) != 0 ? 1u : 0u);
+          umma_commit(&empty[stage]);
+          if (++stage == STAGES) { stage = 0; phase ^= 1; }
+        }
+        if (!ok) break;
+        umma_commit(&tfull[acc]);
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1;
+      }
+      if (*abort_flag) {
+        // every MMA issued so far must finish before TMEM is released
+        umma_commit(teardown);
+        mbar_wait_teardown(teardown, 0);
+      }
+    }
+  } else {
+    const int sp = warp & 3;
+    const int row = sp * 32 + lane;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+      if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, p.err)) break;
+      tc_fence_after();
+      const int m0 = (tile / n_tiles) * BM, n0 = (tile % n_tiles) * BN;
+      const int m = m0 + row;
+      const uint32_t tbase = tmem_base + ((uint32_t)(sp * 32) << 16) + acc * BN;
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        const int n = n0 + c * 32;
+        if (n >= p.N) break;   // uniform across the warp
+        uint32_t r[32];
+        tmem_ld32(tbase + c * 32, r);
+        if (m < p.M) epilogue_chunk<EPI>(p, m, n, r);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
+  }
+}
+
+template <int BN, int EPI>
+static cs_status launch_gemm(const void* A, const void* B, const GemmArgs& args, cudaStream_t stream) {
+  using Cfg = GemmCfg<BN>;
+  CUtensorMap ta, tb;
+  const uint64_t da[2] = {(uint64_t)args.K, (uint64_t)args.M};
+  const uint64_t sa[1] = {(uint64_t)args.K * 2};
+  const uint32_t ba[2] = {64, 128};
+  CS_TRY(make_tmap_bf16(&ta, A, 2, da, sa, ba));
+  const uint64_t db[2] = {(uint64_t)args.K, (uint64_t)args.N};
+  const uint32_t bb[2] = {64, (uint32_t)BN};
+  CS_TRY(make_tmap_bf16(&tb, B, 2, db, sa, bb));
+  auto kern = gemm_tcgen05_kernel<BN, EPI>;
+  CS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
+  const int tiles = ((args.M + 127) / 128) * ((args.N + BN - 1) / BN);
+  const int grid = tiles < num_sms() ? tiles : num_sms();
+  kern<<<grid, 192, Cfg::SMEM, stream>>>(ta, tb, args);
+  CS_LAUNCHED();
+  return CS_OK;
+}
+
+template <int EPI>
+static cs_status dispatch_bn(const void* A, const void* B, const GemmArgs& args, cudaStream_t stream) {
+  if (args.N >= 512) return launch_gemm<256, EPI>(A, B, args, stream);
+  return launch_gemm<128, EPI>(A, B, args, stream);
+}
+
+cs_status gemm_run(const void* A, const void* B, int epi, const GemmArgs& args, cudaStream_t stream) {
+  if (args.M <= 0 || args.N <= 0 || args.K <= 0 || (args.K % 64) != 0) {
+    set_error("gemm: need M, N > 0 and K %% 64 == 0 (M=%d N=%d K=%d)", args.M, args.N, args.K);
+    return CS_ERR_ARG;
+  }
+  if (!A || !B) {
+    set_error("gemm: null operand");
+    return CS_ERR_ARG;
+  }
+  switch (epi) {
+    case CS_EPI_F32: return dispatch_bn<CS_EPI_F32>(A, B, args, stream);
+    case CS_EPI_BF16: return dispatch_bn<CS_EPI_BF16>(A, B, args, stream);
+    case CS_EPI_GELU_BF16: return dispatch_bn<CS_EPI_GELU_BF16>(A, B, args, stream);
+    case CS_EPI_RESID_F32: return dispatch_bn<CS_EPI_RESID_F32>(A, B, args, stream);
+    case CS_EPI_QKV: return dispatch_bn<CS_EPI_QKV>(A, B, args, stream);
+  }
+  set_error("gemm: unknown epilogue %d", epi);
+  return CS_ERR_ARG;
+}
+
+}  // namespace cs
+
+using namespace cs;
+
+extern "C" cs_status cs_gemm_bf16(const void* A, const void* B, int M, int N, int K, int epi, const float* bias,
+                                  const float* gate, void* out, int ldo, int* err, cudaStream_t stream) {
+  CS_REQUIRE(epi != CS_EPI_QKV, "cs_gemm_bf16: use cs_gemm_qkv for the attention-layout epilogue");
+  CS_REQUIRE(out && ldo >= N, "cs_gemm_bf16: need an output with ldo >= N");
+  GemmArgs a{};
+  a.M = M; a.N = N; a.K = K; a.bias = bias; a.gate = gate; a.out = out; a.ldo = ldo; a.err = err;
+  return gemm_run(A, B, epi, a, stream);
+}
+
+extern "C" cs_status cs_gemm_qkv(const void* A, const void* B, int M, int N, int K, const float* bias, int L,
+                                 int d, int heads, int which_base, void* q, void* k, void* vt, int Lv, int* err,
+                                 cudaStream_t stream) {
+  CS_REQUIRE(heads > 0 && d % heads == 0, "cs_gemm_qkv: d must be a multiple of heads");
+  const int hd = d / heads;
+  CS_REQUIRE(hd == 32 || hd == 128, "cs_gemm_qkv: head dim %d not supported (32 or 128)", hd);
+  CS_REQUIRE(L > 0 && M % L == 0 && N % d == 0 && which_base >= 0 && which_base + N / d <= 3,
+             "cs_gemm_qkv: inconsistent M=%d L=%d N=%d d=%d which_base=%d", M, L, N, d, which_base);
+  CS_REQUIRE(Lv >= L && Lv % 8 == 0, "cs_gemm_qkv: Lv must be >= L and a multiple of 8");
+  const int wmax = which_base + N / d;
+  CS_REQUIRE((which_base > 0 || q) && (which_base > 1 || wmax <= 1 || k) && (wmax <= 2 || vt),
+             "cs_gemm_qkv: missing output for a projection");
+  GemmArgs a{};
+  a.M = M; a.N = N; a.K = K; a.bias = bias; a.err = err;
+  a.q = static_cast<__nv_bfloat16*>(q); a.k = static_cast<__nv_bfloat16*>(k);
+  a.vt = static_cast<__nv_bfloat16*>(vt);
+  a.L = L; a.d = d; a.heads = heads; a.hd = hd; a.hd_s = hd < 64 ? 64 : hd; a.Lv = Lv; a.which_base = which_base;
+  return gemm_run(A, B, CS_EPI_QKV, a, stream);
+}

@@ -1,0 +1,58 @@
+"""Host-side checks of the C-ABI library (no GPU needed): it loads, exports every
+symbol the public headers declare, and its host-only queries agree with the layout
+the input generator uses."""
+import os
+import re
+
+import pytest
+
+from paper_2607_23159_gb300 import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    names = set()
+    for h in os.listdir(os.path.join(ROOT, "include")):
+        src = open(os.path.join(ROOT, "include", h)).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        names |= set(re.findall(r"^[A-Za-z_][\w \*]*?\b(cs_\w+)\s*\(", src, flags=re.M))
+    return names
+
+
+@pytest.fixture(scope="module")
+def b():
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_23159_gb300 import binding
+    return binding
+
+
+def test_exports_every_declared_symbol(b):
+    decl = _declared()
+    assert len(decl) >= 20
+    missing = [n for n in decl if not hasattr(b.lib, n)]
+    assert not missing, missing
+    assert decl <= set(b.EXPORTED) | {"cs_last_error"}
+
+
+def test_param_count_matches_generator_layout(b):
+    for m in (synth.TINY, synth.WAN_1_3B, synth.WAN_14B):
+        assert b.param_count(m) == synth.param_count(m)
+
+
+def test_workspace_and_version(b):
+    assert b.lib.cs_version().startswith(b"cachedsearch")
+    assert b.cache_workspace_bytes(4, 2096640) == 4 * 64 * 12
+    assert b.cache_workspace_bytes(0, 10) == 0
+
+
+def test_invalid_config_rejected_on_host(b):
+    import ctypes as C
+    cfg = b.model_config(synth.replace_model(synth.TINY, H=7), 4)   # odd height: no 1x2x2 patches
+    h = C.c_void_p()
+    st = b.lib.cs_init_model(C.byref(cfg), C.byref(h))
+    assert st == b.CS_ERR_ARG and not h.value
+    assert "invalid" in b.last_error()
+    cfg = b.model_config(synth.replace_model(synth.TINY, heads=2), 4)   # head dim 64
+    assert b.lib.cs_init_model(C.byref(cfg), C.byref(h)) == b.CS_ERR_UNSUPPORTED
