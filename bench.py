@@ -1,0 +1,373 @@
+"""Benchmark of the batched cached-search denoising step on GB300.
+
+One bench step = one call of cs_search_step: the cache indicator and decision for all
+N candidates, the DiT forward of the computing subset (30 blocks at the Wan2.1-1.3B
+shape), the fused Delta/Euler update, and (on the last step of a rollout) scoring and
+top-k.  Warm-up steps run on a throwaway search; the timed steps run a fresh search
+from step 1 (a new search starts after T steps).  Metric: candidate-denoising-steps/s.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--tau T]
+  python bench.py --impl reference ...   # the fp64 CPU oracle on a bounded sample
+
+Under torchrun (N > 1) each rank runs an independent search of the same configuration
+(replicas: candidates of different searches never interact), no collective on the data
+path; the reported value is the sum of all ranks' candidate-steps over the slowest
+rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import functools
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "candidate-denoising-steps/sec at Wan2.1-1.3B shape"
+UNIT = "candidate-steps/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="wan1.3b-best-of-4")
+    ap.add_argument("--tau", type=float, default=None)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+# ----------------------------------------------------------------- clocks ----
+
+REASONS = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+
+
+class ClockSampler:
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        q = "clocks.sm,clocks.max.sm,power.draw," + ",".join(f"clocks_event_reasons.{r}" for r in REASONS)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={q}", "--format=csv,noheader,nounits", "-lms", "200", "-i",
+                 str(self.gpu)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.out = ""
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self):
+        rows = []
+        for line in (self.out or "").strip().splitlines():
+            f = [s.strip() for s in line.split(",")]
+            if len(f) < 3 + len(REASONS):
+                continue
+            try:
+                rows.append((float(f[0]), float(f[1]), f[3:3 + len(REASONS)]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        active = sorted({REASONS[i] for _, _, r in rows for i, v in enumerate(r) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": active, "samples": len(rows)}
+
+
+# ------------------------------------------------------------ distributed ----
+
+def dist_setup(gpus):
+    if gpus <= 1 or "RANK" not in os.environ:
+        return 0, 1, 0
+    import torch
+    import torch.distributed as dist
+    rank, world = int(os.environ["RANK"]), int(os.environ["WORLD_SIZE"])
+    local = int(os.environ.get("LOCAL_RANK", rank))
+    torch.cuda.set_device(local)
+    dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(v, world):
+    if world == 1:
+        return v
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([v], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ------------------------------------------------------------ CPU oracle ----
+
+@functools.lru_cache(maxsize=2)
+def _oracle_one_block(m):
+    """One-block oracle model of m's shape and its text K/V (once per prompt, not timed)."""
+    from oracle import cachedsearch_oracle as O
+    from paper_2607_23159_gb300 import synth
+    one = synth.replace_model(m, blocks=1)
+    _, params = synth.make_params(one)
+    dit = O.DiT(one, params)
+    return dit, dit.text_kv(synth.text_context(one))
+
+
+def oracle_sample_seconds(m, rows=512, keys=None, seed=0):
+    """Seconds of the fp64 oracle for one computed candidate-step of model m, from a
+    bounded sample of one block: the K/V projection of `keys` tokens, self-attention of
+    `rows` query rows over those keys, and the rest of the block (projections,
+    cross-attention, FFN) for the `rows` rows.  Each part is scaled to all tokens
+    (attention by both factors) and to all blocks."""
+    from oracle import cachedsearch_oracle as O
+    from paper_2607_23159_gb300 import synth
+    L = m.L
+    rows = min(rows, L)
+    keys = L if keys is None else min(keys, L)
+    dit, kv = _oracle_one_block(m)
+    x = synth.normal(seed, (max(rows, keys), m.d)).astype(np.float64)
+    d, p = m.d, dit.p
+    T0 = time.perf_counter()
+    mods, hm = dit.modulation(0.5)
+    shift1, scale1, gate1, shift2, scale2, gate2 = mods[0]
+    t0 = time.perf_counter()
+    h_k = O.layer_norm(x[:keys]) * (1 + scale1) + shift1
+    kvs = O.linear(h_k, p["blk0.qkv_w"][d:], p["blk0.qkv_b"][d:])
+    t_kv = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    xr = x[:rows]
+    q = O.linear(O.layer_norm(xr) * (1 + scale1) + shift1, p["blk0.qkv_w"][:d], p["blk0.qkv_b"][:d])
+    t_rows = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    sa = O.multi_head_attention(q, kvs[:, :d], kvs[:, d:], m.heads)
+    t_attn = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    xr = xr + gate1 * O.linear(sa, p["blk0.o_w"], p["blk0.o_b"])
+    qc = O.linear(O.layer_norm(xr), p["blk0.cq_w"], p["blk0.cq_b"])
+    xr = xr + O.linear(O.multi_head_attention(qc, kv[0][0], kv[0][1], m.heads), p["blk0.co_w"], p["blk0.co_b"])
+    h = O.layer_norm(xr) * (1 + scale2) + shift2
+    xr = xr + gate2 * O.linear(O.gelu_tanh(O.linear(h, p["blk0.ff1_w"], p["blk0.ff1_b"])), p["blk0.ff2_w"],
+                               p["blk0.ff2_b"])
+    t_rows += time.perf_counter() - t0
+    sample_s = time.perf_counter() - T0
+    per_block = t_kv * (L / keys) + t_rows * (L / rows) + t_attn * (L / rows) * (L / keys)
+    return per_block * m.blocks, sample_s
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(cfg, rows=512):
+    s_per_cs, sample_s = oracle_sample_seconds(cfg.model, rows=rows)
+    rows = min(rows, cfg.model.L)
+    return {"value": 1.0 / s_per_cs, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+            "sample": (f"fp64 numpy oracle, one computed candidate-step of {cfg.name}: 1 of {cfg.model.blocks} "
+                       f"blocks with K/V for all {cfg.model.L} tokens and the rest of the block for {rows} query "
+                       f"rows, scaled to all rows and blocks ({sample_s:.1f} s of CPU work); every "
+                       f"candidate-step counted as computed (skipped steps cost the oracle ~1000x less)")}
+
+
+def run_reference(args, cfg):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    # each step: a bounded sample (128 query rows) of one computed candidate-step
+    for _ in range(args.warmup):
+        oracle_sample_seconds(cfg.model, rows=128, keys=2048)
+    per = []
+    t0 = time.perf_counter()
+    for k in range(args.steps):
+        s, _ = oracle_sample_seconds(cfg.model, rows=128, keys=2048, seed=k)
+        per.append(s)
+    wall = time.perf_counter() - t0
+    val = 1.0 / statistics.mean(per)
+    line = {"impl": "reference", "metric": METRIC, "value": val, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * cfg.N / val, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": cfg.name, "N": cfg.N, "T": cfg.T, "tau": cfg.tau},
+            "cpu_baseline": {"value": val, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                             "sample": (f"per step: fp64 numpy oracle on one block, K/V of "
+                                        f"{min(2048, cfg.model.L)} and query rows {min(128, cfg.model.L)} of "
+                                        f"{cfg.model.L} tokens, scaled to one computed candidate-step of "
+                                        f"{cfg.model.blocks} blocks; {wall:.1f} s total")},
+            "e2e": {"value": val, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------ ours ----
+
+def run_ours(args, cfg):
+    import torch
+    rank, world, local = dist_setup(args.gpus)
+    torch.cuda.set_device(local)
+    from paper_2607_23159_gb300 import binding as B, synth
+    m, N, T = cfg.model, cfg.N, cfg.T
+    tau = cfg.tau if args.tau is None else args.tau
+    flat, _ = synth.make_params(m)
+    x1 = synth.initial_noise(m, range(N)).reshape(N, -1)
+    y = synth.target_latent(m).reshape(-1)
+    model = B.Model(m, N)
+    model.load_weights(flat)
+    del flat
+    model.set_text_context(torch.from_numpy(synth.text_context(m)).cuda())
+    x1_dev = torch.from_numpy(x1).cuda()
+    y_dev = torch.from_numpy(y).cuda()
+    st = B.new_state(N, m.D)
+    skip = torch.zeros(N, dtype=torch.uint8, device="cuda")
+    scores = torch.zeros(N, device="cuda")
+    top = torch.zeros(N, dtype=torch.int32, device="cuda")
+    tgrid = 1.0 - np.arange(T + 1, dtype=np.float64) / T   # t_k = 1 - (k-1)/T
+
+    def reset():
+        st["x"].copy_(x1_dev)
+        st["has_ref"].zero_()
+        st["accum"].zero_()
+
+    def step(i):
+        """search step k = i % T + 1 of the current search (a new search every T steps)."""
+        k = i % T + 1
+        if k == 1:
+            reset()
+        last = k == T
+        n = model.search_step(st, k, T, float(tgrid[k - 1]), float(tgrid[k]), tau, cfg.K_w, cfg.K_c, skip,
+                              target=y_dev if last else None, scores=scores if last else None)
+        if last:
+            B.select_topk(scores, 1, top)
+        return n
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    model.reset_kernel_stats()
+    model.set_profiling(True)
+    launches0 = B.launch_count()
+    computed = 0
+    barrier(world)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record()
+        for i in range(args.steps):
+            computed += step(i)
+        ev1.record()
+        torch.cuda.synchronize()
+        barrier(world)
+    ms_local = ev0.elapsed_time(ev1)
+    launches = B.launch_count() - launches0
+    model.set_profiling(False)
+    stats = {c: model.kernel_stats(c) for c in range(5)}
+    ms = max_over_ranks(ms_local, world)
+    value = N * args.steps * world / (ms / 1e3)
+
+    # end to end through the host-buffer entry point (pinned host latents in, latents + mask out)
+    e2e = None
+    if not args.no_e2e:
+        xh = torch.from_numpy(x1.copy()).pin_memory()
+        skip_h = torch.zeros(N, dtype=torch.uint8).pin_memory()
+        for key in ("has_ref", "accum"):
+            st[key].zero_()
+        barrier(world)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for i in range(args.steps):
+            k = i % T + 1
+            if k == 1:
+                xh.copy_(torch.from_numpy(x1))
+                st["has_ref"].zero_()
+                st["accum"].zero_()
+            model.search_step_host(xh, st, k, T, float(tgrid[k - 1]), float(tgrid[k]), tau, cfg.K_w, cfg.K_c,
+                                   skip_h)
+        torch.cuda.synchronize()
+        barrier(world)
+        e2e_s = max_over_ranks(time.perf_counter() - t0, world)
+        e2e = {"value": N * args.steps * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": int(N * m.D * 4),
+               "d2h_bytes_per_step": int(N * m.D * 4 + N)}
+
+    if rank != 0:
+        return
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except OSError:
+        pass
+    n_sa, ms_sa, fl_sa = stats[B.KC_SELF_ATTN]
+    peak_tf = peaks.get("bf16_tflops_sustained")
+    peak_src = "measured (sustained)" if peak_tf else "fallback (sustained)"
+    peak_tf = peak_tf or 1700.0
+    ach = (fl_sa / n_sa) / (ms_sa / n_sa / 1e3) / 1e12 if n_sa else 0.0
+    n_g, ms_g, fl_g = stats[B.KC_GEMM]
+    n_c, ms_c, by_c = stats[B.KC_CACHE]
+    hbm = peaks.get("hbm_gbs") or 6800.0
+    cache_gbs = by_c / (ms_c / 1e3) / 1e9 if ms_c else 0.0
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded random-init weights and N(0,1) inputs)",
+        "config": {"workload": cfg.name, "N": N, "T": T, "tau": tau, "K_w": cfg.K_w, "K_c": cfg.K_c,
+                   "tokens": m.L, "blocks": m.blocks, "d": m.d, "parallelism": "replicas" if world > 1 else "none",
+                   "l2": "inputs larger than L2 (2.8 GB bf16 weights, GBs of activations per step)"},
+        "roofline": {"kernel": "self-attention (tcgen05 flash attention)", "bound": "tensor", "achieved": ach,
+                     "peak": peak_tf, "peak_source": peak_src, "unit": "TFLOP/s", "frac": ach / peak_tf,
+                     "traffic": None, "launches": n_sa, "avg_ms": ms_sa / n_sa if n_sa else None},
+        "kernels": {
+            "gemm": {"launches": n_g, "ms": ms_g, "tflops": fl_g / (ms_g / 1e3) / 1e12 if ms_g else None,
+                     "frac": (fl_g / (ms_g / 1e3) / 1e12) / peak_tf if ms_g else None},
+            "self_attention": {"launches": n_sa, "ms": ms_sa},
+            "cross_attention": {"launches": stats[B.KC_CROSS_ATTN][0], "ms": stats[B.KC_CROSS_ATTN][1]},
+            "cache_update": {"launches": n_c, "ms": ms_c, "gbs": cache_gbs, "frac_hbm": cache_gbs / hbm},
+            "other": {"launches": stats[B.KC_OTHER][0], "ms": stats[B.KC_OTHER][1]},
+        },
+        "computed_fraction": computed / (N * args.steps),
+        "gpu_launches": launches,
+        "clocks": clk.summary(),
+    }
+    if e2e:
+        line["e2e"] = e2e
+    if not args.no_cpu_baseline and world == 1:
+        line["cpu_baseline"] = cpu_baseline(cfg)
+    print(json.dumps(line), flush=True)
+    model.close()
+
+
+def main():
+    args = parse()
+    from paper_2607_23159_gb300 import synth
+    cfg = synth.CONFIGS[args.config]
+    if args.impl == "reference":
+        run_reference(args, cfg)
+        return
+    import __graft_entry__
+    __graft_entry__.build()
+    run_ours(args, cfg)
+
+
+if __name__ == "__main__":
+    main()
