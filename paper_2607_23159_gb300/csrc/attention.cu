@@ -136,24 +136,23 @@ __global__ void __launch_bounds__(320, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      const uint32_t tS[2] = {tmem_base, tmem_base + 128};
-      const uint32_t tO[2] = {tmem_base + 256, tmem_base + 256 + HD};
-      const uint32_t aQ[2] = {smem_u32(sQ), smem_u32(sQ + Cfg::Q_BYTES)};
-      const uint32_t aP[2] = {smem_u32(sP), smem_u32(sP + Cfg::P_BYTES)};
+      const uint32_t q_base = smem_u32(sQ), p_base = smem_u32(sP);
       auto issue_s = [&](int g, uint32_t kslot) {
+        const uint32_t d = tmem_base + g * 128, a = q_base + g * Cfg::Q_BYTES;
 #pragma unroll
         for (int kk = 0; kk < Cfg::HDS / 16; ++kk) {
           const uint32_t off = (kk >> 2) * Cfg::CH_BYTES + (kk & 3) * 32;
-          umma_bf16_ss(tS[g], sdesc_sw128(aQ[g] + off), sdesc_sw128(kslot + off), Cfg::IDESC_S, kk > 0 ? 1u : 0u);
+          umma_bf16_ss(d, sdesc_sw128(a + off), sdesc_sw128(kslot + off), Cfg::IDESC_S, kk > 0 ? 1u : 0u);
         }
         umma_commit(&s_full[g]);
       };
       auto issue_pv = [&](int g, uint32_t vslot, int j) {
+        const uint32_t d = tmem_base + 256 + g * HD, a = p_base + g * Cfg::P_BYTES;
 #pragma unroll
         for (int kk = 0; kk < Cfg::BKV / 16; ++kk) {
           const uint32_t offa = (kk >> 2) * Cfg::CH_BYTES + (kk & 3) * 32;
           const uint32_t offb = (kk >> 2) * Cfg::VCH_BYTES + (kk & 3) * 32;
-          umma_bf16_ss(tO[g], sdesc_sw128(aP[g] + offa), sdesc_sw128(vslot + offb), Cfg::IDESC_O,
+          umma_bf16_ss(d, sdesc_sw128(a + offa), sdesc_sw128(vslot + offb), Cfg::IDESC_O,
                        (j > 0 || kk > 0) ? 1u : 0u);
         }
         umma_commit(&o_done[g]);
@@ -207,34 +206,43 @@ __global__ void __launch_bounds__(320, 1)
     for (int j = 0; j < nt; ++j) {
       if (!mbar_wait(&s_full[g], j & 1, abort_flag, p.err)) { ok = false; break; }
       tc_fence_after();
-      float x[128];
-#pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        uint32_t u[32];
-        tmem_ld32(tS + c * 32, u);
-#pragma unroll
-        for (int e = 0; e < 32; ++e) x[c * 32 + e] = __uint_as_float(u[e]) * sl2;
-      }
+      uint32_t u[128];
+      tmem_ld128(tS, u);
       const int valid = p.Lk - j * Cfg::BKV;
       if (valid < Cfg::BKV) {
 #pragma unroll
         for (int e = 0; e < 128; ++e)
-          if (e >= valid) x[e] = -INFINITY;
+          if (e >= valid) u[e] = __float_as_uint(-INFINITY);
       }
-      float mx = x[0];
+      // row max of the raw scores: 8 independent chains, then a tree
+      float mx[8];
 #pragma unroll
-      for (int e = 1; e < 128; ++e) mx = fmaxf(mx, x[e]);
-      const float m_new = fmaxf(m_run, mx);
+      for (int q = 0; q < 8; ++q) mx[q] = __uint_as_float(u[q]);
+#pragma unroll
+      for (int e = 8; e < 128; ++e) mx[e & 7] = fmaxf(mx[e & 7], __uint_as_float(u[e]));
+#pragma unroll
+      for (int w = 4; w > 0; w >>= 1)
+#pragma unroll
+        for (int q = 0; q < w; ++q) mx[q] = fmaxf(mx[q], mx[q + w]);
+      const float m_new = fmaxf(m_run, mx[0] * sl2);
       const bool need = (j == 0) || (m_new > m_run + 8.f);
       const bool warp_need = __any_sync(0xffffffffu, need);
       const float m_use = need ? m_new : m_run;
       const float factor = need ? ex2_approx(m_run - m_use) : 1.f;
-      float rs = 0.f;
+      const float nm = -m_use;
+      // p = 2^(s * scale * log2(e) - m), row sum in 8 independent chains
+      float sm[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int e = 0; e < 128; ++e) {
-        x[e] = ex2_approx(x[e] - m_use);
-        rs += x[e];
+        const float pe = ex2_approx(fmaf(__uint_as_float(u[e]), sl2, nm));
+        u[e] = __float_as_uint(pe);
+        sm[e & 7] += pe;
       }
+#pragma unroll
+      for (int w = 4; w > 0; w >>= 1)
+#pragma unroll
+        for (int q = 0; q < w; ++q) sm[q] += sm[q + w];
+      const float rs = sm[0];
       l_run = l_run * factor + rs;
       m_run = m_use;
       if (j > 0) {
@@ -244,26 +252,26 @@ __global__ void __launch_bounds__(320, 1)
         if (warp_need) {
 #pragma unroll 1
           for (int c = 0; c < HD / 32; ++c) {
-            uint32_t u[32];
-            tmem_ld32(tO + c * 32, u);
+            uint32_t o[32];
+            tmem_ld32(tO + c * 32, o);
 #pragma unroll
-            for (int e = 0; e < 32; ++e) u[e] = __float_as_uint(__uint_as_float(u[e]) * factor);
-            tmem_st32(tO + c * 32, u);
+            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * factor);
+            tmem_st32(tO + c * 32, o);
           }
         }
       }
-      // P row -> shared memory, 128-byte swizzle: 16-byte unit u of row r sits at u ^ (r & 7)
+      // P row -> shared memory, 128-byte swizzle: 16-byte unit c8 of row r sits at c8 ^ (r & 7)
 #pragma unroll
       for (int cc = 0; cc < 2; ++cc) {
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const float* v = &x[cc * 64 + u * 8];
+        for (int c8 = 0; c8 < 8; ++c8) {
+          const int b = cc * 64 + c8 * 8;
           uint4 w;
-          w.x = pack_bf16x2(v[0], v[1]);
-          w.y = pack_bf16x2(v[2], v[3]);
-          w.z = pack_bf16x2(v[4], v[5]);
-          w.w = pack_bf16x2(v[6], v[7]);
-          *reinterpret_cast<uint4*>(prow + cc * Cfg::CH_BYTES + ((u ^ (r & 7)) << 4)) = w;
+          w.x = pack_bf16x2(__uint_as_float(u[b + 0]), __uint_as_float(u[b + 1]));
+          w.y = pack_bf16x2(__uint_as_float(u[b + 2]), __uint_as_float(u[b + 3]));
+          w.z = pack_bf16x2(__uint_as_float(u[b + 4]), __uint_as_float(u[b + 5]));
+          w.w = pack_bf16x2(__uint_as_float(u[b + 6]), __uint_as_float(u[b + 7]));
+          *reinterpret_cast<uint4*>(prow + cc * Cfg::CH_BYTES + ((c8 ^ (r & 7)) << 4)) = w;
         }
       }
       fence_proxy_async_smem();

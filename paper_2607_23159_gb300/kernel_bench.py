@@ -1,0 +1,107 @@
+"""Time one of the library's kernels alone at a given shape (CUDA events, warm-up first).
+
+  python -m paper_2607_23159_gb300.kernel_bench attention --batch 1 --L 32760 --heads 12 --hd 128
+  python -m paper_2607_23159_gb300.kernel_bench gemm --M 131040 --N 8960 --K 1536 --epi 2
+  python -m paper_2607_23159_gb300.kernel_bench cache --N 16 --D 2096640
+
+Inputs are random device tensors (the timing does not depend on their values).  Prints
+one JSON line with the average launch time and the achieved TFLOP/s or GB/s.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+
+
+def _time(fn, reps, warmup):
+    import torch
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        fn()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / reps
+
+
+def main():
+    import torch
+    from paper_2607_23159_gb300 import build
+    build.build()
+    from paper_2607_23159_gb300 import binding as B
+    ap = argparse.ArgumentParser()
+    ap.add_argument("kernel", choices=["attention", "gemm", "cache"])
+    ap.add_argument("--batch", type=int, default=1)
+    ap.add_argument("--L", type=int, default=32760)
+    ap.add_argument("--Lk", type=int, default=None)
+    ap.add_argument("--heads", type=int, default=12)
+    ap.add_argument("--hd", type=int, default=128)
+    ap.add_argument("--M", type=int, default=131040)
+    ap.add_argument("--N", type=int, default=1536)
+    ap.add_argument("--K", type=int, default=1536)
+    ap.add_argument("--epi", type=int, default=1)
+    ap.add_argument("--D", type=int, default=2096640)
+    ap.add_argument("--skip-frac", type=float, default=1.0)
+    ap.add_argument("--reps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=2)
+    a = ap.parse_args()
+    dev = "cuda"
+    bf = torch.bfloat16
+    out = {"kernel": a.kernel}
+    if a.kernel == "attention":
+        Lk = a.Lk or a.L
+        hds = max(a.hd, 64)
+        BH = a.batch * a.heads
+        q = torch.randn(BH, a.L, hds, device=dev).to(bf)
+        k = torch.randn(BH, Lk, hds, device=dev).to(bf)
+        if hds > a.hd:
+            q[:, :, a.hd:] = 0
+            k[:, :, a.hd:] = 0
+        Ls = (Lk + 7) // 8 * 8
+        vt = torch.randn(BH, a.hd, Ls, device=dev).to(bf)
+        o = torch.empty(a.batch, a.L, a.heads * a.hd, device=dev, dtype=bf)
+        ms = _time(lambda: B.attention(q, k, vt, o, a.batch, a.heads, a.L, Lk, a.hd, Ls, False), a.reps, a.warmup)
+        flops = 4.0 * BH * a.L * Lk * a.hd
+        out.update(shape=dict(batch=a.batch, L=a.L, Lk=Lk, heads=a.heads, hd=a.hd), ms=ms,
+                   tflops=flops / (ms / 1e3) / 1e12)
+    elif a.kernel == "gemm":
+        A = torch.randn(a.M, a.K, device=dev).to(bf)
+        W = (torch.randn(a.N, a.K, device=dev) * 0.05).to(bf)
+        bias = torch.zeros(a.N, device=dev)
+        if a.epi in (B.EPI_F32, B.EPI_RESID_F32):
+            C = torch.zeros(a.M, a.N, device=dev)
+        else:
+            C = torch.empty(a.M, a.N, device=dev, dtype=bf)
+        ms = _time(lambda: B.gemm(A, W, a.epi, C, bias=bias), a.reps, a.warmup)
+        out.update(shape=dict(M=a.M, N=a.N, K=a.K, epi=a.epi), ms=ms,
+                   tflops=2.0 * a.M * a.N * a.K / (ms / 1e3) / 1e12)
+    else:
+        N, D = a.N, a.D
+        st = B.new_state(N, D)
+        st["x"].normal_()
+        st["x_ref"].copy_(st["x"] * 0.99)
+        st["delta"].normal_()
+        st["has_ref"].fill_(1)
+        v = torch.randn(N, D, device=dev)
+        ws = torch.zeros(B.cache_workspace_bytes(N, D) // 4 + 1, device=dev)
+        skip = torch.zeros(N, dtype=torch.uint8, device=dev)
+        idx = torch.zeros(N, dtype=torch.int32, device=dev)
+        nc = torch.zeros(1, dtype=torch.int32, device=dev)
+        force = (torch.rand(N, device=dev) >= a.skip_frac).to(torch.uint8)
+
+        def run():
+            B.cache_decide(st["x"], st["x_ref"], st["accum"], st["has_ref"], 20, 50, 0.1, 5, 5, skip, idx, nc, ws,
+                           force=force)
+            B.cache_apply(st["x"], st["x_ref"], st["delta"], v, skip, 0.6, 0.58)
+        ms = _time(run, a.reps, a.warmup)
+        n_skip = int((force == 0).sum())
+        byts = (n_skip * 16.0 + (N - n_skip) * 24.0) * D
+        out.update(shape=dict(N=N, D=D, skipped=n_skip), ms=ms, gbs=byts / (ms / 1e3) / 1e9)
+    print(json.dumps(out), flush=True)
+
+
+if __name__ == "__main__":
+    main()
