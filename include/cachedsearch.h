@@ -120,6 +120,28 @@ cs_status cs_cache_decide(const float* x_dev, const float* x_ref_dev, float* acc
                           const uint8_t* force_compute_dev, uint8_t* skip_mask_dev, int32_t* compute_idx_dev,
                           int32_t* n_compute_dev, void* workspace_dev, int* err_dev, cudaStream_t stream);
 
+/* Allocation-free form of cs_cache_decide, for callers that cannot allocate device
+ * memory: a serving runtime whose memory pool owns the whole device after start-up, or
+ * host code that must not let an allocation synchronise the device mid-step.  It takes
+ * no workspace; the partial sums live in a fixed array compiled into the library (one
+ * per GPU that loads it, kept until the process exits, 64 KB).  The paper has no
+ * counterpart: this is a deployment convenience of this library.
+ *   Limits: N <= CS_NOALLOC_MAX_N candidates and D <= CS_NOALLOC_MAX_CHUNKS * 32768
+ *   elements per candidate; larger sizes return CS_ERR_ARG with a message, nothing runs.
+ *   The first call on a device looks up the array's device address (cudaGetSymbolAddress)
+ *   with that device current; make that first call before any stream capture.
+ *   All calls on a device share the array: calls that overlap on the GPU (other streams
+ *   or threads) race and must be serialised by the caller.  Each call writes every
+ *   partial it reads, so nothing from a previous call needs clearing.
+ * Arguments, results and errors are those of cs_cache_decide. */
+#define CS_NOALLOC_MAX_N 64
+#define CS_NOALLOC_MAX_CHUNKS 128
+cs_status cs_cache_decide_noalloc(const float* x_dev, const float* x_ref_dev, float* accum_dev,
+                                  uint8_t* has_ref_dev, int N, long long D, int step_k, int T, float tau,
+                                  int K_w, int K_c, const uint8_t* force_compute_dev, uint8_t* skip_mask_dev,
+                                  int32_t* compute_idx_dev, int32_t* n_compute_dev, int* err_dev,
+                                  cudaStream_t stream);
+
 /* Cache rule, part 2, fused with the Euler update (Eq. delta, Eq. skip, Eq. euler),
  * h = t_next - t_cur:
  *   skipped:  x += h (x + Delta)

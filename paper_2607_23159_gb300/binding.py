@@ -49,6 +49,7 @@ _SIGS = {
     "cs_dit_forward": (I, [P, P, P, I, F, P, P]),
     "cs_cache_workspace_bytes": (SZ, [I, LL]),
     "cs_cache_decide": (I, [P, P, P, P, I, LL, I, I, F, I, I, P, P, P, P, P, P, P]),
+    "cs_cache_decide_noalloc": (I, [P, P, P, P, I, LL, I, I, F, I, I, P, P, P, P, P, P]),
     "cs_cache_apply": (I, [P, P, P, P, P, I, LL, F, F, P, P, P, P]),
     "cs_search_step": (I, [P, P, P, P, P, P, I, I, I, F, F, F, I, I, P, P, P, P, P, P]),
     "cs_search_step_host": (I, [P, P, P, P, P, P, I, I, I, F, F, F, I, I, P, P, P]),
@@ -149,6 +150,16 @@ def cache_decide(x, x_ref, accum, has_ref, step_k, T, tau, K_w, K_c, skip_mask, 
     check(lib.cs_cache_decide(_ptr(x), _ptr(x_ref), _ptr(accum), _ptr(has_ref), N, Dn, step_k, T, tau, K_w, K_c,
                               _ptr(force), _ptr(skip_mask), _ptr(compute_idx), _ptr(n_compute), _ptr(workspace),
                               _ptr(err), _stream(stream)))
+
+
+def cache_decide_noalloc(x, x_ref, accum, has_ref, step_k, T, tau, K_w, K_c, skip_mask, compute_idx, n_compute,
+                         force=None, err=None, stream=None):
+    """cs_cache_decide without a workspace (fixed scratch inside the library)."""
+    N = x.shape[0]
+    Dn = x[0].numel()
+    check(lib.cs_cache_decide_noalloc(_ptr(x), _ptr(x_ref), _ptr(accum), _ptr(has_ref), N, Dn, step_k, T, tau, K_w,
+                                      K_c, _ptr(force), _ptr(skip_mask), _ptr(compute_idx), _ptr(n_compute),
+                                      _ptr(err), _stream(stream)))
 
 
 def cache_apply(x, x_ref, delta, v, skip_mask, t_cur, t_next, workspace=None, target=None, scores=None,

@@ -13,6 +13,7 @@
 // present), so a candidate's numbers are the same whatever batch it is in.
 #include <cmath>
 #include <cstdint>
+#include <mutex>
 
 #include "common.cuh"
 #include "ptx.cuh"
@@ -390,6 +391,78 @@ extern "C" cs_status cs_beam_refill(const float* sx, const float* sr, const floa
   const int slots = keep * (children + 1);
   beam_refill_kernel<<<dim3(cache_chunks(D), slots), kCacheThreads, 0, stream>>>(
       sx, sr, sd, sa, sh, dx, dr, dd, da, dh, surv, children, sigma, noise, D);
+  CS_LAUNCHED();
+  return CS_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of cs_cache_decide.
+//
+// Some callers cannot call cudaMalloc: a serving runtime whose memory pool has taken
+// all device memory at start-up, or host code that must never let an allocation
+// synchronise the device in the middle of a step.  For them the drift partial sums
+// live in a fixed array compiled into this library instead of a caller workspace.
+// The array exists once per GPU that loads the library and is held until the process
+// exits; every call on that GPU shares it, so calls that overlap on the GPU (two
+// streams, or two threads) race and must be serialised by the caller.  Each call
+// writes every partial it later reads, so nothing carried over from an earlier call
+// is ever used and nothing needs clearing.
+// ---------------------------------------------------------------------------
+namespace cs {
+
+constexpr int kStaticMaxN = CS_NOALLOC_MAX_N;
+constexpr int kStaticMaxChunks = CS_NOALLOC_MAX_CHUNKS;
+static __device__ __align__(256) float g_decide_scratch[kStaticMaxN * kStaticMaxChunks * 2];
+
+static std::mutex g_scratch_mu;
+static float* g_scratch_ptr[256] = {};   // device address of g_decide_scratch, per device ordinal
+
+// Device address of the scratch array on the current device (looked up once per device).
+static cs_status static_scratch(float** out) {
+  int dev = 0;
+  CS_CUDA(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= 256) {
+    set_error("cs_cache_decide_noalloc: device ordinal %d out of range", dev);
+    return CS_ERR_ARG;
+  }
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_ptr[dev]) {
+    void* p = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&p, g_decide_scratch);
+    if (e != cudaSuccess || !p) {
+      set_error("cs_cache_decide_noalloc: cudaGetSymbolAddress failed on device %d: %s", dev, cudaGetErrorString(e));
+      return CS_ERR_CUDA;
+    }
+    g_scratch_ptr[dev] = static_cast<float*>(p);
+  }
+  *out = g_scratch_ptr[dev];
+  return CS_OK;
+}
+
+}  // namespace cs
+
+extern "C" cs_status cs_cache_decide_noalloc(const float* x, const float* x_ref, float* accum, uint8_t* has_ref,
+                                             int N, long long D, int step_k, int T, float tau, int K_w, int K_c,
+                                             const uint8_t* force, uint8_t* skip_mask, int32_t* idx,
+                                             int32_t* n_compute, int* err, cudaStream_t stream) {
+  CS_REQUIRE(N > 0 && D > 0, "cs_cache_decide_noalloc: need N > 0 and D > 0 (N=%d D=%lld)", N, D);
+  CS_REQUIRE(N <= kStaticMaxN, "cs_cache_decide_noalloc: N=%d exceeds the fixed scratch limit of %d candidates", N,
+             kStaticMaxN);
+  CS_REQUIRE(cache_chunks(D) <= kStaticMaxChunks,
+             "cs_cache_decide_noalloc: D=%lld exceeds the fixed scratch limit of %lld elements per candidate", D,
+             (long long)kStaticMaxChunks * kChunkElems);
+  CS_REQUIRE(x && x_ref && accum && has_ref && skip_mask && idx && n_compute, "cs_cache_decide_noalloc: null pointer");
+  CS_REQUIRE(step_k >= 1 && step_k <= T, "cs_cache_decide_noalloc: step %d outside 1..T=%d", step_k, T);
+  float* partials = nullptr;
+  CS_TRY(static_scratch(&partials));
+  const int nch = cache_chunks(D);
+  const int wf = window_forced(step_k, T, K_w, K_c) ? 1 : 0;
+  if (!wf) {
+    drift_partials_kernel<<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, has_ref, D, wf, partials);
+    CS_LAUNCHED();
+  }
+  decide_finalize_kernel<<<1, 256, N, stream>>>(partials, nch, accum, has_ref, N, wf, tau, force, skip_mask, idx,
+                                                n_compute, err);
   CS_LAUNCHED();
   return CS_OK;
 }
