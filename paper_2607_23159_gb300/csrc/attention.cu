@@ -2,18 +2,21 @@
 // the DiT blocks).  One CTA takes 256 query rows of one (batch item, head) as two
 // 128-row tiles A and B and streams the keys in tiles of 128:
 //
-//   warp 0      TMA producer: Q once, then K_j and V_j^T tiles through a 3-slot ring
-//   warp 1      TMEM allocator + MMA issuer, in the order
-//                 S_A(0) S_B(0) | PV_A(j) S_A(j+1) PV_B(j) S_B(j+1) | ...
-//               so that the tensor core works on one tile while the other's softmax runs
-//   warps 2..5  softmax of tile A, warps 6..9 softmax of tile B: one query row per
-//               thread; S row from TMEM, online max/sum in log2 units with lazy O
-//               rescaling (only when the running max grows by more than 8), P as bf16
-//               into shared memory in the 128-byte-swizzled K-major layout the MMA reads
+//   warp 0       TMA producer: Q once, then K_j and V_j^T tiles through a 4-slot ring
+//   warp 1       TMEM allocator + MMA issuer, in the order
+//                  S_A(0) S_B(0) | PV_A(j) S_A(j+1) PV_B(j) S_B(j+1) | ...
+//                so that the tensor core works on one tile while the other's softmax runs
+//   warps 2..9   softmax of tile A, warps 10..17 softmax of tile B.  Two threads share a
+//                query row (warps w and w+4 read the same TMEM lanes): each takes 64 of the
+//                128 keys, the two exchange their row maxima through shared memory and a
+//                named barrier, and keep separate partial row sums until the end.  Online
+//                softmax in log2 units with lazy O rescaling (only when the running max
+//                grows by more than 8).  P is written back to TMEM as bf16 over the
+//                thread's own S columns and fed to the PV MMA as the TMEM A operand.
 //
-// TMEM (512 columns): S_A [0,128), S_B [128,256), O_A [256, 256+hd), O_B [256+hd, 256+2hd).
-// S = Q K^T and O += P V are both M=128 tcgen05.mma with operands in shared memory;
-// V is stored transposed (V^T [hd][keys]) so that it is a K-major B operand.
+// TMEM (512 columns): S_A [0,128), S_B [128,256) (P_g aliases the first 32 columns of
+// each 64-key half of S_g), O_A [256, 256+hd), O_B [256+hd, 256+2hd).  V is stored
+// transposed (V^T [hd][keys]) so that it is a K-major B operand in shared memory.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -33,7 +36,7 @@ struct AttnArgs {
 template <int HD>
 struct AttnCfg {
   static constexpr int HDS = HD < 64 ? 64 : HD;   // Q/K row length in shared memory
-  static constexpr int BQ = 128, BKV = 128;
+  static constexpr int BKV = 128;
   static constexpr int QCH = HDS / 64;             // 64-wide chunks of a Q/K row
   static constexpr int CH_BYTES = 128 * 64 * 2;    // one [128 x 64] bf16 chunk
   static constexpr int Q_BYTES = QCH * CH_BYTES;   // one 128-row Q tile
@@ -41,32 +44,36 @@ struct AttnCfg {
   static constexpr int VCH_BYTES = HD * 64 * 2;    // one [hd x 64 keys] chunk of V^T
   static constexpr int V_BYTES = 2 * VCH_BYTES;
   static constexpr int SLOT = K_BYTES > V_BYTES ? K_BYTES : V_BYTES;
-  static constexpr int NSLOT = 3;
-  static constexpr int P_BYTES = 2 * CH_BYTES;     // 128 rows x 128 keys
-  static constexpr int SMEM = 2 * Q_BYTES + NSLOT * SLOT + 2 * P_BYTES + 1024 + 256;
+  static constexpr int NSLOT = 4;
+  static constexpr int XBUF_BYTES = 2 * 2 * 2 * 128 * 4;   // [parity][tile][half][row] floats
+  static constexpr int SMEM = 2 * Q_BYTES + NSLOT * SLOT + XBUF_BYTES + 1024 + 256;
+  static constexpr int THREADS = 18 * 32;
+  static constexpr int OCOLS = HD >= 64 ? HD / 2 : HD;   // O columns each half-thread owns
   static constexpr uint32_t IDESC_S = idesc_bf16_f32(128, BKV);
   static constexpr uint32_t IDESC_O = idesc_bf16_f32(128, HD);
 };
 
 template <int HD>
-__global__ void __launch_bounds__(320, 1)
+__global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
     attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                         const __grid_constant__ CUtensorMap tmV, const AttnArgs p) {
   using Cfg = AttnCfg<HD>;
+  constexpr int NS = Cfg::NSLOT;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;                                   // [2][Q_BYTES]
-  uint8_t* sKV = sQ + 2 * Cfg::Q_BYTES;                 // [3][SLOT]
-  uint8_t* sP = sKV + Cfg::NSLOT * Cfg::SLOT;           // [2][P_BYTES]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + 2 * Cfg::P_BYTES);
+  uint8_t* sKV = sQ + 2 * Cfg::Q_BYTES;                 // [NSLOT][SLOT]
+  float* xbuf = reinterpret_cast<float*>(sKV + NS * Cfg::SLOT);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(xbuf) + Cfg::XBUF_BYTES);
   uint64_t* q_full = bars;
-  uint64_t* kv_full = bars + 1;       // [3]
-  uint64_t* kv_empty = bars + 4;      // [3]
-  uint64_t* s_full = bars + 7;        // [2]
-  uint64_t* p_full = bars + 9;        // [2]
-  uint64_t* o_done = bars + 11;       // [2]
-  uint64_t* teardown = bars + 13;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 14);
+  uint64_t* kv_full = bars + 1;            // [NS]
+  uint64_t* kv_empty = kv_full + NS;       // [NS]
+  uint64_t* s_full = kv_empty + NS;        // [2]
+  uint64_t* p_full = s_full + 2;           // [2]
+  uint64_t* o_done = p_full + 2;           // [2]
+  uint64_t* teardown = o_done + 2;
+  uint64_t* xbar = teardown + 1;           // [2][4]: the two warps of one row quarter
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(xbar + 8);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -78,16 +85,17 @@ __global__ void __launch_bounds__(320, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int s = 0; s < 3; ++s) {
+    for (int s = 0; s < NS; ++s) {
       mbar_init(&kv_full[s], 1);
       mbar_init(&kv_empty[s], 1);
     }
     for (int g = 0; g < 2; ++g) {
       mbar_init(&s_full[g], 1);
-      mbar_init(&p_full[g], 128);
+      mbar_init(&p_full[g], 256);
       mbar_init(&o_done[g], 1);
     }
     mbar_init(teardown, 1);
+    for (int i = 0; i < 8; ++i) mbar_init(&xbar[i], 64);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -112,8 +120,8 @@ __global__ void __launch_bounds__(320, 1)
           tma_load_3d(sQ + g * Cfg::Q_BYTES + c * Cfg::CH_BYTES, &tmQ, q_full, c * 64, q0 + g * 128, bh);
       int issued = 0;
       for (int s = 0; s < 2 * nt; ++s) {
-        const int slot = s % 3;
-        const uint32_t ph = (s / 3) & 1;
+        const int slot = s % NS;
+        const uint32_t ph = (s / NS) & 1;
         if (!mbar_wait(&kv_empty[slot], ph ^ 1, abort_flag, p.err)) break;
         uint8_t* dst = sKV + slot * Cfg::SLOT;
         const int j = s >> 1;
@@ -130,13 +138,14 @@ __global__ void __launch_bounds__(320, 1)
       }
       if (*abort_flag) {
         mbar_wait_teardown(q_full, 0);
-        for (int s = issued - 3 < 0 ? 0 : issued - 3; s < issued; ++s) mbar_wait_teardown(&kv_full[s % 3], (s / 3) & 1);
+        for (int s = issued - NS < 0 ? 0 : issued - NS; s < issued; ++s)
+          mbar_wait_teardown(&kv_full[s % NS], (s / NS) & 1);
       }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      const uint32_t q_base = smem_u32(sQ), p_base = smem_u32(sP);
+      const uint32_t q_base = smem_u32(sQ);
       auto issue_s = [&](int g, uint32_t kslot) {
         const uint32_t d = tmem_base + g * 128, a = q_base + g * Cfg::Q_BYTES;
 #pragma unroll
@@ -147,17 +156,17 @@ __global__ void __launch_bounds__(320, 1)
         umma_commit(&s_full[g]);
       };
       auto issue_pv = [&](int g, uint32_t vslot, int j) {
-        const uint32_t d = tmem_base + 256 + g * HD, a = p_base + g * Cfg::P_BYTES;
+        const uint32_t d = tmem_base + 256 + g * HD;
 #pragma unroll
         for (int kk = 0; kk < Cfg::BKV / 16; ++kk) {
-          const uint32_t offa = (kk >> 2) * Cfg::CH_BYTES + (kk & 3) * 32;
+          // keys 16kk..16kk+15: half kk/4, packed bf16 pairs at columns 8*(kk%4) of that half
+          const uint32_t a = tmem_base + g * 128 + (kk >> 2) * 64 + (kk & 3) * 8;
           const uint32_t offb = (kk >> 2) * Cfg::VCH_BYTES + (kk & 3) * 32;
-          umma_bf16_ss(d, sdesc_sw128(a + offa), sdesc_sw128(vslot + offb), Cfg::IDESC_O,
-                       (j > 0 || kk > 0) ? 1u : 0u);
+          umma_bf16_ts(d, a, sdesc_sw128(vslot + offb), Cfg::IDESC_O, (j > 0 || kk > 0) ? 1u : 0u);
         }
         umma_commit(&o_done[g]);
       };
-      auto slot_addr = [&](int s) { return smem_u32(sKV + (s % 3) * Cfg::SLOT); };
+      auto slot_addr = [&](int s) { return smem_u32(sKV + (s % NS) * Cfg::SLOT); };
       bool ok = mbar_wait(q_full, 0, abort_flag, p.err);
       if (ok) ok = mbar_wait(&kv_full[0], 0, abort_flag, p.err);
       if (ok) {
@@ -168,22 +177,22 @@ __global__ void __launch_bounds__(320, 1)
       }
       for (int j = 0; ok && j < nt; ++j) {
         const int sv = 2 * j + 1, sk = 2 * j + 2;
-        if (!mbar_wait(&kv_full[sv % 3], (sv / 3) & 1, abort_flag, p.err)) break;
+        if (!mbar_wait(&kv_full[sv % NS], (sv / NS) & 1, abort_flag, p.err)) break;
         if (!mbar_wait(&p_full[0], j & 1, abort_flag, p.err)) break;
         tc_fence_after();
         issue_pv(0, slot_addr(sv), j);
         if (j + 1 < nt) {
-          if (!mbar_wait(&kv_full[sk % 3], (sk / 3) & 1, abort_flag, p.err)) break;
+          if (!mbar_wait(&kv_full[sk % NS], (sk / NS) & 1, abort_flag, p.err)) break;
           tc_fence_after();
           issue_s(0, slot_addr(sk));
         }
         if (!mbar_wait(&p_full[1], j & 1, abort_flag, p.err)) break;
         tc_fence_after();
         issue_pv(1, slot_addr(sv), j);
-        umma_commit(&kv_empty[sv % 3]);
+        umma_commit(&kv_empty[sv % NS]);
         if (j + 1 < nt) {
           issue_s(1, slot_addr(sk));
-          umma_commit(&kv_empty[sk % 3]);
+          umma_commit(&kv_empty[sk % NS]);
         }
       }
       if (*abort_flag) {
@@ -193,65 +202,78 @@ __global__ void __launch_bounds__(320, 1)
     }
   } else {
     // ------------------------------------------------------------ softmax
-    const int g = (warp - 2) >> 2;          // 0: tile A (warps 2..5), 1: tile B (warps 6..9)
-    const int sp = warp & 3;                // TMEM lane quarter this warp may access
-    const int r = sp * 32 + lane;           // query row inside the tile
-    const uint32_t lane_off = (uint32_t)(sp * 32) << 16;
-    const uint32_t tS = tmem_base + lane_off + g * 128;
-    const uint32_t tO = tmem_base + lane_off + 256 + g * HD;
-    uint8_t* prow = sP + g * Cfg::P_BYTES + r * 128;
+    const int sw = warp - 2;
+    const int g = sw >> 3;                  // query tile: 0 = A (warps 2..9), 1 = B (warps 10..17)
+    const int h = (sw >> 2) & 1;            // which 64 keys of each tile this thread takes
+    const int qtr = warp & 3;               // TMEM lane quarter this warp may access
+    const int r = qtr * 32 + lane;          // query row inside the tile
+    uint64_t* pair_bar = &xbar[g * 4 + qtr];   // the two warps of one row quarter
+    const uint32_t lane_off = (uint32_t)(qtr * 32) << 16;
+    const uint32_t tS = tmem_base + lane_off + g * 128 + h * 64;
+    const uint32_t tO = tmem_base + lane_off + 256 + g * HD + h * Cfg::OCOLS;
+    const bool owns_o = (HD >= 64) || (h == 0);
     const float sl2 = p.scale_log2;
+    const uint64_t sc2 = f2_pack(sl2, sl2);
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     for (int j = 0; j < nt; ++j) {
-      if (!mbar_wait(&s_full[g], j & 1, abort_flag, p.err)) { ok = false; break; }
+      if (!__all_sync(0xffffffffu, mbar_wait(&s_full[g], j & 1, abort_flag, p.err))) { ok = false; break; }
       tc_fence_after();
-      uint32_t u[128];
-      tmem_ld128(tS, u);
-      const int valid = p.Lk - j * Cfg::BKV;
-      if (valid < Cfg::BKV) {
+      uint32_t u[64];
+      tmem_ld64(tS, u);
+      const int valid = p.Lk - j * Cfg::BKV - h * 64;
+      if (valid < 64) {
 #pragma unroll
-        for (int e = 0; e < 128; ++e)
+        for (int e = 0; e < 64; ++e)
           if (e >= valid) u[e] = __float_as_uint(-INFINITY);
       }
-      // row max of the raw scores: 8 independent chains, then a tree
-      float mx[8];
+      float mx[4];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) mx[q] = __uint_as_float(u[q]);
+      for (int q = 0; q < 4; ++q) mx[q] = __uint_as_float(u[q]);
 #pragma unroll
-      for (int e = 8; e < 128; ++e) mx[e & 7] = fmaxf(mx[e & 7], __uint_as_float(u[e]));
+      for (int e = 4; e < 64; e += 8) {
 #pragma unroll
-      for (int w = 4; w > 0; w >>= 1)
-#pragma unroll
-        for (int q = 0; q < w; ++q) mx[q] = fmaxf(mx[q], mx[q + w]);
-      const float m_new = fmaxf(m_run, mx[0] * sl2);
+        for (int q = 0; q < 4; ++q) mx[q] = fmax3(mx[q], __uint_as_float(u[e + 2 * q]), __uint_as_float(u[e + 2 * q + 1]));
+      }
+      float* xb = xbuf + ((j & 1) * 2 + g) * 256;
+      xb[h * 128 + r] = fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
+      mbar_arrive(pair_bar);   // release: the partner sees this row max after its wait
+      if (!__all_sync(0xffffffffu, mbar_wait(pair_bar, j & 1, abort_flag, p.err))) { ok = false; break; }
+      const float rmax = fmaxf(xb[r], xb[128 + r]);
+      const float m_new = fmaxf(m_run, rmax * sl2);
       const bool need = (j == 0) || (m_new > m_run + 8.f);
       const bool warp_need = __any_sync(0xffffffffu, need);
       const float m_use = need ? m_new : m_run;
       const float factor = need ? ex2_approx(m_run - m_use) : 1.f;
-      const float nm = -m_use;
-      // p = 2^(s * scale * log2(e) - m), row sum in 8 independent chains
-      float sm[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      const uint64_t nm2 = f2_pack(-m_use, -m_use);
+      // p = 2^(s * scale * log2(e) - m) on pairs; P packed as bf16 pairs in place
+      uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-      for (int e = 0; e < 128; ++e) {
-        const float pe = ex2_approx(fmaf(__uint_as_float(u[e]), sl2, nm));
-        u[e] = __float_as_uint(pe);
-        sm[e & 7] += pe;
+      for (int i = 0; i < 32; ++i) {
+        float a, b;
+        f2_unpack(f2_fma(f2_pack(__uint_as_float(u[2 * i]), __uint_as_float(u[2 * i + 1])), sc2, nm2), a, b);
+        a = ex2_approx(a);
+        b = ex2_approx(b);
+        acc[i & 3] = f2_add(acc[i & 3], f2_pack(a, b));
+        u[i] = pack_bf16x2(a, b);
       }
-#pragma unroll
-      for (int w = 4; w > 0; w >>= 1)
-#pragma unroll
-        for (int q = 0; q < w; ++q) sm[q] += sm[q + w];
-      const float rs = sm[0];
-      l_run = l_run * factor + rs;
+      float s0, s1, s2, s3, s4, s5, s6, s7;
+      f2_unpack(acc[0], s0, s1);
+      f2_unpack(acc[1], s2, s3);
+      f2_unpack(acc[2], s4, s5);
+      f2_unpack(acc[3], s6, s7);
+      l_run = l_run * factor + (((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7)));
       m_run = m_use;
       if (j > 0) {
         // PV of the previous tile must be done before O is rescaled and P overwritten
-        if (!mbar_wait(&o_done[g], (j - 1) & 1, abort_flag, p.err)) { ok = false; break; }
+        if (!__all_sync(0xffffffffu, mbar_wait(&o_done[g], (j - 1) & 1, abort_flag, p.err))) {
+          ok = false;
+          break;
+        }
         tc_fence_after();
-        if (warp_need) {
+        if (warp_need && owns_o) {
 #pragma unroll 1
-          for (int c = 0; c < HD / 32; ++c) {
+          for (int c = 0; c < Cfg::OCOLS / 32; ++c) {
             uint32_t o[32];
             tmem_ld32(tO + c * 32, o);
 #pragma unroll
@@ -260,32 +282,30 @@ __global__ void __launch_bounds__(320, 1)
           }
         }
       }
-      // P row -> shared memory, 128-byte swizzle: 16-byte unit c8 of row r sits at c8 ^ (r & 7)
+      uint32_t pk[32];
 #pragma unroll
-      for (int cc = 0; cc < 2; ++cc) {
-#pragma unroll
-        for (int c8 = 0; c8 < 8; ++c8) {
-          const int b = cc * 64 + c8 * 8;
-          uint4 w;
-          w.x = pack_bf16x2(__uint_as_float(u[b + 0]), __uint_as_float(u[b + 1]));
-          w.y = pack_bf16x2(__uint_as_float(u[b + 2]), __uint_as_float(u[b + 3]));
-          w.z = pack_bf16x2(__uint_as_float(u[b + 4]), __uint_as_float(u[b + 5]));
-          w.w = pack_bf16x2(__uint_as_float(u[b + 6]), __uint_as_float(u[b + 7]));
-          *reinterpret_cast<uint4*>(prow + cc * Cfg::CH_BYTES + ((c8 ^ (r & 7)) << 4)) = w;
-        }
-      }
-      fence_proxy_async_smem();
+      for (int i = 0; i < 32; ++i) pk[i] = u[i];
+      tmem_st32(tS, pk);
       tc_fence_before();
       mbar_arrive(&p_full[g]);
     }
-    if (ok && mbar_wait(&o_done[g], (nt - 1) & 1, abort_flag, p.err)) {
+    // final: row sum of both halves, then O / l -> bf16
+    float* xb = xbuf + ((nt & 1) * 2 + g) * 256;
+    xb[h * 128 + r] = l_run;
+    if (ok) {
+      mbar_arrive(pair_bar);
+      ok = __all_sync(0xffffffffu, mbar_wait(pair_bar, nt & 1, abort_flag, p.err));
+    }
+    const float l_tot = xb[r] + xb[128 + r];
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&o_done[g], (nt - 1) & 1, abort_flag, p.err));
+    if (ok && owns_o) {
       tc_fence_after();
       const int q = q0 + g * 128 + r;
-      const float inv_l = 1.f / l_run;
+      const float inv_l = 1.f / l_tot;
       const int d = p.heads * HD;
-      __nv_bfloat16* orow = p.o + ((long long)jb * p.Lq + q) * d + head * HD;
+      __nv_bfloat16* orow = p.o + ((long long)jb * p.Lq + q) * d + head * HD + h * Cfg::OCOLS;
 #pragma unroll 1
-      for (int c = 0; c < HD / 32; ++c) {
+      for (int c = 0; c < Cfg::OCOLS / 32; ++c) {
         uint32_t u[32];
         tmem_ld32(tO + c * 32, u);
         if (q < p.Lq) {
@@ -343,7 +363,7 @@ static cs_status launch_attn(const void* q, const void* k, const void* vt, void*
   auto kern = attn_tcgen05_kernel<HD>;
   CS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
   dim3 grid((Lq + 255) / 256, BH);
-  kern<<<grid, 320, Cfg::SMEM, stream>>>(tq, tk, tv, a);
+  kern<<<grid, Cfg::THREADS, Cfg::SMEM, stream>>>(tq, tk, tv, a);
   CS_LAUNCHED();
   return CS_OK;
 }

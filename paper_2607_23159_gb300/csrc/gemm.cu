@@ -253,7 +253,7 @@ __global__ void __launch_bounds__(192, 1)
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
-      if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, p.err)) break;
+      if (!__all_sync(0xffffffffu, mbar_wait(&tfull[acc], acc_phase, abort_flag, p.err))) break;
       tc_fence_after();
       const int m0 = (tile / n_tiles) * BM, n0 = (tile % n_tiles) * BN;
       const int m = m0 + row;
