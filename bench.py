@@ -31,6 +31,9 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "candidate-denoising-steps/sec at Wan2.1-1.3B shape"
+# DRAM bytes (read + write) of one self-attention launch per (candidate, head) at 32760
+# tokens, hd 128, from the ncu capture in profiles/attn_tcgen05_hd128_L32760.md
+ATTN_DRAM_BYTES_PER_HEAD_L32760 = 387.7e6 / 12
 UNIT = "candidate-steps/s"
 
 
@@ -323,6 +326,8 @@ def run_ours(args, cfg):
     peak_src = "measured (sustained)" if peak_tf else "fallback (sustained)"
     peak_tf = peak_tf or 1700.0
     ach = (fl_sa / n_sa) / (ms_sa / n_sa / 1e3) / 1e12 if n_sa else 0.0
+    heads_per_launch = (fl_sa / n_sa) / (4.0 * m.L * m.L * m.hd) if n_sa else 0.0
+    traffic = heads_per_launch * ATTN_DRAM_BYTES_PER_HEAD_L32760 if (m.L == 32760 and m.hd == 128) else None
     n_g, ms_g, fl_g = stats[B.KC_GEMM]
     n_c, ms_c, by_c = stats[B.KC_CACHE]
     hbm = peaks.get("hbm_gbs") or 6800.0
@@ -336,7 +341,7 @@ def run_ours(args, cfg):
                    "l2": "inputs larger than L2 (2.8 GB bf16 weights, GBs of activations per step)"},
         "roofline": {"kernel": "self-attention (tcgen05 flash attention)", "bound": "tensor", "achieved": ach,
                      "peak": peak_tf, "peak_source": peak_src, "unit": "TFLOP/s", "frac": ach / peak_tf,
-                     "traffic": None, "launches": n_sa, "avg_ms": ms_sa / n_sa if n_sa else None},
+                     "traffic": traffic, "launches": n_sa, "avg_ms": ms_sa / n_sa if n_sa else None},
         "kernels": {
             "gemm": {"launches": n_g, "ms": ms_g, "tflops": fl_g / (ms_g / 1e3) / 1e12 if ms_g else None,
                      "frac": (fl_g / (ms_g / 1e3) / 1e12) / peak_tf if ms_g else None},
