@@ -231,7 +231,7 @@ def run_ours(args, cfg):
     import torch
     rank, world, local = dist_setup(args.gpus)
     torch.cuda.set_device(local)
-    from paper_2607_23159_gb300 import binding as B, synth
+    from paper_2607_23159_gb300 import binding as B, search as S, synth
     m, N, T = cfg.model, cfg.N, cfg.T
     tau = cfg.tau if args.tau is None else args.tau
     flat, _ = synth.make_params(m)
@@ -243,27 +243,27 @@ def run_ours(args, cfg):
     model.set_text_context(torch.from_numpy(synth.text_context(m)).cuda())
     x1_dev = torch.from_numpy(x1).cuda()
     y_dev = torch.from_numpy(y).cuda()
-    st = B.new_state(N, m.D)
-    skip = torch.zeros(N, dtype=torch.uint8, device="cuda")
-    scores = torch.zeros(N, device="cuda")
-    top = torch.zeros(N, dtype=torch.int32, device="cuda")
-    tgrid = 1.0 - np.arange(T + 1, dtype=np.float64) / T   # t_k = 1 - (k-1)/T
-
-    def reset():
-        st["x"].copy_(x1_dev)
-        st["has_ref"].zero_()
-        st["accum"].zero_()
+    srch = S.Search(model, N, target=y_dev)
+    beam = cfg.beam_every > 0
+    noise = ([torch.from_numpy(synth.beam_noise(m, r, cfg.beam_keep, cfg.beam_children).reshape(-1, m.D)).cuda()
+              for r in range((T - 1) // cfg.beam_every)] if beam else None)
+    rnd = [0]
 
     def step(i):
-        """search step k = i % T + 1 of the current search (a new search every T steps)."""
+        """search step k = i % T + 1 of the current search (a new search every T steps);
+        beam workloads rescore and refill every beam_every steps."""
         k = i % T + 1
         if k == 1:
-            reset()
+            srch.reset(x1_dev)
+            rnd[0] = 0
         last = k == T
-        n = model.search_step(st, k, T, float(tgrid[k - 1]), float(tgrid[k]), tau, cfg.K_w, cfg.K_c, skip,
-                              target=y_dev if last else None, scores=scores if last else None)
+        rescore = beam and k % cfg.beam_every == 0 and not last
+        n = srch.step(k, T, tau, cfg.K_w, cfg.K_c, score=last or rescore)
+        if rescore:
+            srch.refill(srch.select(cfg.beam_keep).clone(), cfg.beam_children, cfg.beam_sigma, noise[rnd[0]])
+            rnd[0] += 1
         if last:
-            B.select_topk(scores, 1, top)
+            srch.select(1)
         return n
 
     for i in range(args.warmup):
@@ -292,11 +292,11 @@ def run_ours(args, cfg):
 
     # end to end through the host-buffer entry point (pinned host latents in, latents + mask out)
     e2e = None
-    if not args.no_e2e:
+    tgrid = S.time_grid(T)
+    if not args.no_e2e and not beam:   # host-buffer path: plain best-of-N steps
         xh = torch.from_numpy(x1.copy()).pin_memory()
         skip_h = torch.zeros(N, dtype=torch.uint8).pin_memory()
-        for key in ("has_ref", "accum"):
-            st[key].zero_()
+        st = B.new_state(N, m.D)
         barrier(world)
         torch.cuda.synchronize()
         t0 = time.perf_counter()

@@ -357,8 +357,72 @@ def beam_refill(states, xs, survivors, children, sigma, noise):
             cp = CacheState(None if st.delta is None else st.delta.copy(),
                             None if st.x_ref is None else st.x_ref.copy(), st.a)
             x = np.asarray(xs[src], np.float64).copy()
-            if j > 0:
+            if j > 0:  # children only exist when children > 0
                 x = x + sigma * np.asarray(noise[p * children + j - 1], np.float64)
             new_states.append(cp)
             new_x.append(x)
     return new_states, np.stack(new_x)
+
+
+# ---------------------------------------------------------------------------
+# search variants built on the same step
+# ---------------------------------------------------------------------------
+
+def static_schedule(k, T, K_w, K_c, every):
+    """Static uniform-schedule baseline (Sec. 3.1, Properties): warmup and cooldown steps
+    compute; between them a step computes when (k - K_w) is a multiple of ``every``."""
+    if k <= K_w or k > T - K_c:
+        return True
+    return (k - K_w) % every == 0
+
+
+def rollout_static(x1, T, K_w, K_c, every, velocity_fn_t):
+    """Cached rollout whose decisions follow :func:`static_schedule` (the indicator is
+    still accumulated but does not decide)."""
+    mask = np.array([static_schedule(k, T, K_w, K_c, every) for k in range(1, T + 1)])
+    return rollout(x1, T, 1e30, K_w, K_c, velocity_fn_t, force_mask=mask)
+
+
+def commit(x1, T, velocity_fn_t):
+    """Algorithm 1, commit branch: regenerate the chosen seed at full compute, G(c, s)."""
+    return rollout_uncached(x1, T, velocity_fn_t)
+
+
+def beam_search(x1s, T, tau, K_w, K_c, velocity_fn_t, target, every, keep, children, sigma, noise_for_round):
+    """Beam-style cached search (workload reading; the paper's closest step is the
+    prune-and-continue composition of Sec. abl-stack): every ``every`` steps (before the
+    last) score the x0 estimate, keep the top ``keep`` and refill each with ``children``
+    perturbed copies (:func:`beam_refill`).  Returns (final scores, final latents, masks)."""
+    states = [CacheState() for _ in range(len(x1s))]
+    xs = np.asarray(x1s, np.float64)
+    masks, r = [], 0
+    for k in range(1, T + 1):
+        rescore = (k % every == 0 and k < T) or k == T
+        xs, skipped, _, sc = search_step(states, xs, k, T, tau, K_w, K_c, velocity_fn_t,
+                                         target=target if rescore else None)
+        masks.append(skipped)
+        if k % every == 0 and k < T:
+            surv = topk(sc, keep)
+            states, xs = beam_refill(states, xs, list(surv), children, sigma, noise_for_round(r))
+            r += 1
+    return sc, xs, np.array(masks)
+
+
+def pruned_search(x1s, T, tau, K_w, K_c, velocity_fn_t, target, prune_step, keep):
+    """Cached search with mid-trajectory pruning (Sec. abl-stack): all candidates run
+    cached to ``prune_step``, are scored on the sampler's x0 estimate, and only the top
+    ``keep`` continue to step T.  Returns (winner's original index, final scores of the
+    survivors, survivor original indices, final latents of the survivors)."""
+    states = [CacheState() for _ in range(len(x1s))]
+    xs = np.asarray(x1s, np.float64)
+    ids = np.arange(len(x1s))
+    for k in range(1, T + 1):
+        prune = k == prune_step
+        xs, _, _, sc = search_step(states, xs, k, T, tau, K_w, K_c, velocity_fn_t,
+                                   target=target if (prune or k == T) else None)
+        if prune:
+            surv = topk(sc, keep)
+            states, xs = beam_refill(states, xs, list(surv), 0, 0.0, None)
+            ids = ids[surv]
+    best = int(topk(sc, 1)[0])
+    return int(ids[best]), sc, ids, xs

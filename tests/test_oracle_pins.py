@@ -315,3 +315,40 @@ def test_dit_zero_blocks_reduce_to_head_of_embedding():
     sd = np.sqrt(tok.var(1, keepdims=True) + 1e-6)
     out = ((tok - mu) / sd * (1 + hm[1]) + hm[0]) @ m.p["head_w"].T
     np.testing.assert_allclose(O.patchify(m.velocity(x, t, kv)), out, atol=1e-12)
+
+
+# ------------------------------------------------------------ search variants ---
+
+def test_static_schedule_hand_example_and_every_one_is_uncached():
+    got = [O.static_schedule(k, 12, 2, 2, 3) for k in range(1, 13)]
+    # warmup 1-2, cooldown 11-12, in between k - 2 in {3, 6} -> k = 5, 8
+    assert [int(g) for g in got] == [1, 1, 0, 0, 1, 0, 0, 1, 0, 0, 1, 1]
+    cfg, m = _tiny_model(blocks=1)
+    kv = m.text_kv(synth.text_context(cfg))
+    x1 = synth.initial_noise(cfg, [0])[0]
+    vel = lambda x, t: m.velocity(x, t, kv)
+    xs, comp, _ = O.rollout_static(x1, 6, 1, 1, 1, vel)
+    assert comp.all() and np.array_equal(xs, O.rollout_uncached(x1, 6, vel))
+    assert np.array_equal(O.commit(x1, 6, vel), O.rollout_uncached(x1, 6, vel))
+
+
+def test_beam_and_pruned_search_degenerate_cases():
+    cfg, m = _tiny_model(blocks=1)
+    kv = m.text_kv(synth.text_context(cfg))
+    x1s = synth.initial_noise(cfg, range(4))
+    y = synth.target_latent(cfg)
+    vel = lambda x, t: m.velocity(x, t, kv)
+    T = 6
+    i_star, sc, _, _ = O.cached_search(x1s, T, 0.1, 1, 1, vel, y)
+    # keep everything, no children: the beam only permutes slots
+    sb, _, _ = O.beam_search(x1s, T, 0.1, 1, 1, vel, y, every=2, keep=4, children=0, sigma=0.0,
+                             noise_for_round=lambda r: None)
+    np.testing.assert_allclose(np.sort(sb), np.sort(sc), rtol=1e-12)
+    # sigma = 0 children are exact copies of their parent
+    sb, xb, _ = O.beam_search(x1s, T, 0.1, 1, 1, vel, y, every=3, keep=2, children=1, sigma=0.0,
+                              noise_for_round=lambda r: np.ones((2, *x1s.shape[1:])))
+    assert np.array_equal(xb[0], xb[1]) and np.array_equal(xb[2], xb[3])
+    # pruning that keeps every candidate picks the same winner as the plain search
+    win, sp, ids, _ = O.pruned_search(x1s, T, 0.1, 1, 1, vel, y, prune_step=3, keep=4)
+    assert win == i_star
+    np.testing.assert_allclose(np.sort(sp), np.sort(sc), rtol=1e-12)
