@@ -92,6 +92,11 @@ cs_status cs_load_weights(cs_model* model, const float* params, size_t count, in
  * by all candidates, Algorithm 1). */
 cs_status cs_set_text_context(cs_model* model, const float* ctx_dev, cudaStream_t stream);
 
+/* Classifier-free guidance (Eq. cfg): the unconditional ("empty prompt") text context
+ * ctx_dev [Lt][d_text], projected like cs_set_text_context into a second K/V set per
+ * block.  Needed by cs_search_step_cfg. */
+cs_status cs_set_null_text_context(cs_model* model, const float* ctx_dev, cudaStream_t stream);
+
 /* Velocity of a compacted subset: for j < n_c, v_dev[idx[j]] = v_theta(x_dev[idx[j]], t, c)
  * (Sec. 2).  idx_dev: int32 [n_c] candidate indices (device); n_c <= max_batch.  Rows of
  * v_dev not named in idx are left untouched. */
@@ -151,6 +156,31 @@ cs_status cs_cache_decide_noalloc(const float* x_dev, const float* x_ref_dev, fl
 cs_status cs_cache_apply(float* x_dev, float* x_ref_dev, float* delta_dev, const float* v_dev,
                          const uint8_t* skip_mask_dev, int N, long long D, float t_cur, float t_next,
                          const float* target_dev, float* scores_dev, void* workspace_dev, cudaStream_t stream);
+
+/* Guided forms (Eq. cfg with per-branch cache state, Sec. 3.1): each candidate i has two
+ * cache states, row i (conditional branch) and row N + i (unconditional branch), that
+ * share its latent x_i and decide independently.  x_ref, delta: [2N][D]; accum, has_ref,
+ * force_compute, skip_mask: [2N]; compute_idx: [2N] state rows; workspace:
+ * cs_cache_workspace_bytes(2N, D).  The apply step combines the two branch velocities
+ * (computed v_b, or x + Delta_b when skipped) as v_u + w (v_c - v_u) and takes the Euler
+ * step with it; scores use that combined velocity in the x0 estimate. */
+cs_status cs_cache_decide_cfg(const float* x_dev, const float* x_ref_dev, float* accum_dev, uint8_t* has_ref_dev,
+                              int N, long long D, int step_k, int T, float tau, int K_w, int K_c,
+                              const uint8_t* force_compute_dev, uint8_t* skip_mask_dev, int32_t* compute_idx_dev,
+                              int32_t* n_compute_dev, void* workspace_dev, int* err_dev, cudaStream_t stream);
+cs_status cs_cache_apply_cfg(float* x_dev, float* x_ref_dev, float* delta_dev, const float* v_dev,
+                             const uint8_t* skip_mask_dev, int N, long long D, float t_cur, float t_next, float w,
+                             const float* target_dev, float* scores_dev, void* workspace_dev, cudaStream_t stream);
+
+/* One guided denoising step of N candidates: both branches' decisions, one DiT forward
+ * of all computing branch items (conditional items use the prompt's K/V, unconditional
+ * items the null context's), then the guided update.  2N <= max_batch.  Same state
+ * conventions as the guided forms above; *n_computed counts branch items. */
+cs_status cs_search_step_cfg(cs_model* model, float* x_dev, float* x_ref_dev, float* delta_dev, float* accum_dev,
+                             uint8_t* has_ref_dev, int N, int step_k, int T, float t_cur, float t_next, float tau,
+                             int K_w, int K_c, float guidance, const uint8_t* force_compute_dev,
+                             uint8_t* skip_mask_dev, const float* target_dev, float* scores_dev, int* n_computed,
+                             cudaStream_t stream);
 
 /* One denoising step of N candidates (the unit of work of the search):
  * cs_cache_decide, then cs_dit_forward on the computing subset, then cs_cache_apply.

@@ -426,3 +426,39 @@ def pruned_search(x1s, T, tau, K_w, K_c, velocity_fn_t, target, prune_step, keep
             ids = ids[surv]
     best = int(topk(sc, 1)[0])
     return int(ids[best]), sc, ids, xs
+
+
+# ---------------------------------------------------------------------------
+# classifier-free guidance with per-branch cache state (Eq. cfg; Sec. 3.1, per-branch state)
+# ---------------------------------------------------------------------------
+
+def cfg_combine(v_uncond, v_cond, w):
+    """``v(x, t, 0) + w (v(x, t, c) - v(x, t, 0))`` (Eq. cfg)."""
+    return v_uncond + w * (v_cond - v_uncond)
+
+
+def search_step_cfg(states_c, states_u, xs, k, T, tau, K_w, K_c, vel_cond_t, vel_uncond_t, w,
+                    force_c=None, force_u=None, target=None):
+    """One guided Euler step of every candidate.  Each branch keeps its own cache state
+    and takes its own decision on the same latent input (Sec. 3.1, per-branch cache
+    state); the two velocities (computed or ``x + Delta_b``) are combined by Eq. cfg and
+    the Euler step uses the combination.  Returns (x_next, skipped_c, skipped_u, scores)."""
+    t = time_grid(T)
+    out, sk_c, sk_u, vs = [], [], [], []
+    for i in range(len(xs)):
+        x = np.asarray(xs[i], np.float64)
+        fc = None if force_c is None else bool(force_c[i])
+        fu = None if force_u is None else bool(force_u[i])
+        v_c, comp_c, _ = wrapper_call(states_c[i], x, k, T, tau, K_w, K_c, lambda z: vel_cond_t(z, t[k - 1]), fc)
+        v_u, comp_u, _ = wrapper_call(states_u[i], x, k, T, tau, K_w, K_c, lambda z: vel_uncond_t(z, t[k - 1]), fu)
+        v = cfg_combine(v_u, v_c, w)
+        out.append(euler(x, t[k - 1], t[k], v))
+        vs.append(v)
+        sk_c.append(not comp_c)
+        sk_u.append(not comp_u)
+    out = np.stack(out)
+    scores = None
+    if target is not None:
+        x0 = out - t[k] * np.stack(vs)
+        scores = np.array([score(x0[i], target) for i in range(len(xs))])
+    return out, np.array(sk_c), np.array(sk_u), scores

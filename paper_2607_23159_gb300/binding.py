@@ -46,7 +46,11 @@ _SIGS = {
     "cs_destroy_model": (I, [P]),
     "cs_load_weights": (I, [P, P, SZ, I, P]),
     "cs_set_text_context": (I, [P, P, P]),
+    "cs_set_null_text_context": (I, [P, P, P]),
     "cs_dit_forward": (I, [P, P, P, I, F, P, P]),
+    "cs_cache_decide_cfg": (I, [P, P, P, P, I, LL, I, I, F, I, I, P, P, P, P, P, P, P]),
+    "cs_cache_apply_cfg": (I, [P, P, P, P, P, I, LL, F, F, F, P, P, P, P]),
+    "cs_search_step_cfg": (I, [P, P, P, P, P, P, I, I, I, F, F, F, I, I, F, P, P, P, P, P, P]),
     "cs_cache_workspace_bytes": (SZ, [I, LL]),
     "cs_cache_decide": (I, [P, P, P, P, I, LL, I, I, F, I, I, P, P, P, P, P, P, P]),
     "cs_cache_decide_noalloc": (I, [P, P, P, P, I, LL, I, I, F, I, I, P, P, P, P, P, P]),
@@ -224,6 +228,20 @@ class Model:
     def set_text_context(self, ctx, stream=None):
         check(lib.cs_set_text_context(self.h, _ptr(ctx), _stream(stream)))
 
+    def set_null_text_context(self, ctx, stream=None):
+        check(lib.cs_set_null_text_context(self.h, _ptr(ctx), _stream(stream)))
+
+    def search_step_cfg(self, st, k, T, t_cur, t_next, tau, K_w, K_c, w, skip_mask, force=None, target=None,
+                        scores=None, stream=None) -> int:
+        """Guided step; st from new_state_cfg (x [N, D], branch states [2N, ...])."""
+        n = C.c_int(0)
+        N = st["x"].shape[0]
+        check(lib.cs_search_step_cfg(self.h, _ptr(st["x"]), _ptr(st["x_ref"]), _ptr(st["delta"]),
+                                     _ptr(st["accum"]), _ptr(st["has_ref"]), N, k, T, t_cur, t_next, tau, K_w, K_c,
+                                     w, _ptr(force), _ptr(skip_mask), _ptr(target), _ptr(scores), C.byref(n),
+                                     _stream(stream)))
+        return n.value
+
     def dit_forward(self, x, idx, n_c, t, v, stream=None):
         check(lib.cs_dit_forward(self.h, _ptr(x), _ptr(idx), n_c, t, _ptr(v), _stream(stream)))
 
@@ -260,6 +278,15 @@ class Model:
 
     def reset_kernel_stats(self):
         check(lib.cs_reset_kernel_stats(self.h))
+
+
+def new_state_cfg(N: int, D: int, device="cuda"):
+    """Zeroed guided-search state: latents [N, D]; two branch cache states per candidate
+    (rows i and N + i)."""
+    import torch
+    st = new_state(2 * N, D, device)
+    st["x"] = torch.zeros(N, D, dtype=torch.float32, device=device)
+    return st
 
 
 def new_state(N: int, D: int, device="cuda"):

@@ -47,8 +47,8 @@ struct cs_model {
   std::vector<BlockW> blk;
   float** mod_offs_dev = nullptr;
   // text K/V (per block) and its scratch
-  bf16 *ktext, *vttext, *txt1, *txt, *ctx_bf16;
-  bool text_set = false;
+  bf16 *ktext, *vttext, *txt1, *txt, *ctx_bf16;   // ktext [block][set][H][Lt][hd_s], vttext [block][set][H][hd][Ltv]
+  bool text_set = false, null_text_set = false;
   // workspace (one allocation)
   void* ws = nullptr;
   bf16 *tok, *hbuf, *obuf, *q, *k, *vt, *fbuf;
@@ -125,6 +125,15 @@ cs_status attention(cs_model* m, int cls, const void* q, const void* k, const vo
   return record_end(m, cls, s, ev, 4.0 * B * m->cfg.heads * (double)Lq * Lk * m->hd);
 }
 
+cs_status cross_attention(cs_model* m, const void* q, const void* k, const void* vt, void* o, int B, int Lq, int Lk,
+                          int Lkv_stride, int kv_sets, const int32_t* idx, int x_rows, cudaStream_t s) {
+  cudaEvent_t ev[2];
+  CS_TRY(record_begin(m, 1, s, ev));
+  CS_TRY(cs::attention_run(q, k, vt, o, B, m->cfg.heads, Lq, Lk, m->hd, Lkv_stride, 1, kv_sets,
+                           kv_sets > 1 ? idx : nullptr, x_rows, m->err, s));
+  return record_end(m, 1, s, ev, 4.0 * B * m->cfg.heads * (double)Lq * Lk * m->hd);
+}
+
 bool valid_cfg(const cs_model_config* c) {
   if (!c) return false;
   if (c->C <= 0 || c->F <= 0 || c->H <= 0 || c->W <= 0 || (c->H & 1) || (c->W & 1)) return false;
@@ -196,7 +205,7 @@ extern "C" cs_status cs_init_model(const cs_model_config* cfg, cs_model** out) {
     addb(&w.ff2_w, d * F); addf(&w.ff2_b, d);
   }
   // text K/V cache + text scratch
-  const size_t kt = nb * cfg->heads * (size_t)cfg->Lt * m->hd_s, vtt = nb * cfg->heads * (size_t)hd * m->Ltv;
+  const size_t kt = 2 * nb * cfg->heads * (size_t)cfg->Lt * m->hd_s, vtt = 2 * nb * cfg->heads * (size_t)hd * m->Ltv;
   addb(&m->ktext, kt);
   addb(&m->vttext, vtt);
   addb(&m->txt1, (size_t)cfg->Lt * d);
@@ -351,8 +360,9 @@ extern "C" cs_status cs_load_weights(cs_model* m, const float* params, size_t co
   return CS_OK;
 }
 
-extern "C" cs_status cs_set_text_context(cs_model* m, const float* ctx, cudaStream_t s) {
-  CS_REQUIRE(m && ctx, "cs_set_text_context: null pointer");
+// Project a text context into K/V set `set` of every block (0: the prompt, 1: the
+// unconditional context of classifier-free guidance).
+static cs_status project_text(cs_model* m, const float* ctx, int set, cudaStream_t s) {
   const cs_model_config& c = m->cfg;
   const int d = c.d;
   CS_TRY(cs::to_bf16_pad(ctx, c.Lt, c.d_text, c.d_text, m->ctx_bf16, s));
@@ -363,18 +373,29 @@ extern "C" cs_status cs_set_text_context(cs_model* m, const float* ctx, cudaStre
   for (int b = 0; b < c.blocks; ++b) {
     // per block: [K | V] = text W_ckv^T + b_ckv, laid out per head (K) and transposed (V)
     CS_TRY(gemm_qkv(m, m->txt, m->blk[b].ckv_w, c.Lt, 2 * d, d, m->blk[b].ckv_b, c.Lt, 1, nullptr,
-                    m->ktext + b * kt, m->vttext + b * vtt, m->Ltv, s));
+                    m->ktext + (2 * b + set) * kt, m->vttext + (2 * b + set) * vtt, m->Ltv, s));
   }
+  return CS_OK;
+}
+
+extern "C" cs_status cs_set_text_context(cs_model* m, const float* ctx, cudaStream_t s) {
+  CS_REQUIRE(m && ctx, "cs_set_text_context: null pointer");
+  CS_TRY(project_text(m, ctx, 0, s));
   m->text_set = true;
   return CS_OK;
 }
 
-extern "C" cs_status cs_dit_forward(cs_model* m, const float* x, const int32_t* idx, int n_c, float t, float* v,
-                                    cudaStream_t s) {
-  CS_REQUIRE(m && x && idx && v, "cs_dit_forward: null pointer");
-  CS_REQUIRE(n_c >= 0 && n_c <= m->cfg.max_batch, "cs_dit_forward: n_c=%d outside 0..max_batch=%d", n_c,
-             m->cfg.max_batch);
-  CS_REQUIRE(m->text_set, "cs_dit_forward: call cs_set_text_context first");
+extern "C" cs_status cs_set_null_text_context(cs_model* m, const float* ctx, cudaStream_t s) {
+  CS_REQUIRE(m && ctx, "cs_set_null_text_context: null pointer");
+  CS_TRY(project_text(m, ctx, 1, s));
+  m->null_text_set = true;
+  return CS_OK;
+}
+
+// DiT forward of items j < n_c: latent row idx[j] % x_rows, cross-attention K/V set
+// idx[j] / x_rows (kv_sets = 2 for guidance), velocity written to v[idx[j]].
+static cs_status dit_forward_impl(cs_model* m, const float* x, const int32_t* idx, int n_c, int x_rows, int kv_sets,
+                                  float t, float* v, cudaStream_t s) {
   if (n_c == 0) return CS_OK;
   const cs_model_config& c = m->cfg;
   const int d = c.d, L = m->L, M = n_c * L;
@@ -383,7 +404,7 @@ extern "C" cs_status cs_dit_forward(cs_model* m, const float* x, const int32_t* 
   cs::CondWeights cw{d, c.f_dim, c.blocks, m->time_w1, m->time_w2, m->mod_w, m->head_mod_w,
                      m->time_b1, m->time_b2, m->mod_b, m->head_mod_b, m->mod_offs_dev};
   CS_TRY(cs::timestep_conditioning(cw, t, m->cond_scratch, m->mods, m->hmod, s));
-  CS_TRY(cs::patchify(x, idx, n_c, c.C, c.F, c.H, c.W, m->Kp, m->tok, s));
+  CS_TRY(cs::patchify(x, idx, n_c, x_rows, c.C, c.F, c.H, c.W, m->Kp, m->tok, s));
   CS_TRY(record_end(m, 4, s, ev, 0.0));
   CS_TRY(gemm(m, m->tok, m->patch_w, CS_EPI_F32, m->patch_b, nullptr, m->resid, d, M, d, m->Kp, s));
   const size_t kt = (size_t)c.heads * c.Lt * m->hd_s, vtt = (size_t)c.heads * m->hd * m->Ltv;
@@ -402,7 +423,8 @@ extern "C" cs_status cs_dit_forward(cs_model* m, const float* x, const int32_t* 
     CS_TRY(cs::layernorm_modulate(m->resid, nullptr, nullptr, m->hbuf, M, d, s));
     CS_TRY(record_end(m, 4, s, ev, 0.0));
     CS_TRY(gemm_qkv(m, m->hbuf, w.cq_w, M, d, d, w.cq_b, L, 0, m->q, nullptr, nullptr, m->Lv, s));
-    CS_TRY(attention(m, 1, m->q, m->ktext + b * kt, m->vttext + b * vtt, m->obuf, n_c, L, c.Lt, m->Ltv, 1, s));
+    CS_TRY(cross_attention(m, m->q, m->ktext + 2 * b * kt, m->vttext + 2 * b * vtt, m->obuf, n_c, L, c.Lt, m->Ltv,
+                           kv_sets, idx, x_rows, s));
     CS_TRY(gemm(m, m->obuf, w.co_w, CS_EPI_RESID_F32, w.co_b, nullptr, m->resid, d, M, d, d, s));
     // h = LN(x)(1 + scale2) + shift2 ; x += gate2 * FFN(h)
     CS_TRY(record_begin(m, 4, s, ev));
@@ -420,6 +442,15 @@ extern "C" cs_status cs_dit_forward(cs_model* m, const float* x, const int32_t* 
   CS_TRY(cs::unpatchify(m->hout, idx, n_c, c.C, c.F, c.H, c.W, v, s));
   CS_TRY(record_end(m, 4, s, ev, 0.0));
   return CS_OK;
+}
+
+extern "C" cs_status cs_dit_forward(cs_model* m, const float* x, const int32_t* idx, int n_c, float t, float* v,
+                                    cudaStream_t s) {
+  CS_REQUIRE(m && x && idx && v, "cs_dit_forward: null pointer");
+  CS_REQUIRE(n_c >= 0 && n_c <= m->cfg.max_batch, "cs_dit_forward: n_c=%d outside 0..max_batch=%d", n_c,
+             m->cfg.max_batch);
+  CS_REQUIRE(m->text_set, "cs_dit_forward: call cs_set_text_context first");
+  return dit_forward_impl(m, x, idx, n_c, 1 << 30, 1, t, v, s);
 }
 
 static cs_status step_impl(cs_model* m, float* x, float* x_ref, float* delta, float* accum, uint8_t* has_ref, int N,
@@ -447,7 +478,7 @@ static cs_status step_impl(cs_model* m, float* x, float* x_ref, float* delta, fl
     return (cs_status)code;
   }
   if (n_out) *n_out = n_c;
-  CS_TRY(cs_dit_forward(m, x, m->idx, n_c, t_cur, m->v, s));
+  CS_TRY(dit_forward_impl(m, x, m->idx, n_c, N, 1, t_cur, m->v, s));
   CS_TRY(record_begin(m, 3, s, ev));
   CS_TRY(cs_cache_apply(x, x_ref, delta, m->v, skip, N, D, t_cur, t_next, target, scores, m->cache_ws, s));
   // algorithmic bytes of indicator + update (each tensor read or written once):
@@ -466,6 +497,44 @@ extern "C" cs_status cs_search_step(cs_model* m, float* x, float* x_ref, float* 
                                     float* scores, int* n_computed, cudaStream_t s) {
   return step_impl(m, x, x_ref, delta, accum, has_ref, N, k, T, t_cur, t_next, tau, K_w, K_c, force, skip, target,
                    scores, n_computed, s);
+}
+
+extern "C" cs_status cs_search_step_cfg(cs_model* m, float* x, float* x_ref, float* delta, float* accum,
+                                        uint8_t* has_ref, int N, int k, int T, float t_cur, float t_next, float tau,
+                                        int K_w, int K_c, float w, const uint8_t* force, uint8_t* skip,
+                                        const float* target, float* scores, int* n_out, cudaStream_t s) {
+  CS_REQUIRE(m && x && x_ref && delta && accum && has_ref && skip, "cs_search_step_cfg: null pointer");
+  CS_REQUIRE(N > 0 && 2 * N <= m->cfg.max_batch, "cs_search_step_cfg: 2N=%d exceeds max_batch=%d", 2 * N,
+             m->cfg.max_batch);
+  CS_REQUIRE(m->text_set && m->null_text_set, "cs_search_step_cfg: set both text contexts first");
+  CS_REQUIRE(!target || scores, "cs_search_step_cfg: scoring needs scores");
+  const long long D = m->D;
+  cudaEvent_t ev[2];
+  const bool wf = k <= K_w || k > T - K_c;
+  CS_TRY(record_begin(m, 3, s, ev));
+  CS_TRY(cs_cache_decide_cfg(x, x_ref, accum, has_ref, N, D, k, T, tau, K_w, K_c, force, skip, m->idx, m->n_compute,
+                             m->cache_ws, m->err, s));
+  CS_TRY(record_end(m, 3, s, ev, 0.0));
+  CS_CUDA(cudaMemcpyAsync(m->n_host, m->n_compute, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
+  CS_CUDA(cudaMemcpyAsync(m->n_host + 1, m->err, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
+  CS_CUDA(cudaStreamSynchronize(s));
+  const int n_c = m->n_host[0];
+  if (m->n_host[1] != 0) {
+    cs::set_error("cs_search_step_cfg: device error %d recorded before step %d", m->n_host[1], k);
+    const int code = m->n_host[1];
+    cudaMemsetAsync(m->err, 0, sizeof(int), s);
+    return (cs_status)code;
+  }
+  if (n_out) *n_out = n_c;
+  // branch items: state rows < N are conditional (K/V set 0), rows >= N unconditional (set 1)
+  CS_TRY(dit_forward_impl(m, x, m->idx, n_c, N, 2, t_cur, m->v, s));
+  CS_TRY(record_begin(m, 3, s, ev));
+  CS_TRY(cs_cache_apply_cfg(x, x_ref, delta, m->v, skip, N, D, t_cur, t_next, w, target, scores, m->cache_ws, s));
+  const double skipped = 2.0 * N - n_c;
+  double bytes = 4.0 * D * N * 2 + skipped * 8.0 * D + n_c * (wf ? 12.0 : 16.0) * D;   // x in/out + per branch
+  if (target) bytes += 4.0 * D * N;
+  CS_TRY(record_end(m, 3, s, ev, bytes));
+  return CS_OK;
 }
 
 extern "C" cs_status cs_search_step_host(cs_model* m, float* x_host, float* x_ref, float* delta, float* accum,

@@ -21,6 +21,7 @@
 #include <cuda_bf16.h>
 
 #include "common.cuh"
+#include "elementwise.h"
 #include "ptx.cuh"
 #include "tma_host.h"
 
@@ -28,6 +29,8 @@ namespace cs {
 
 struct AttnArgs {
   int B, heads, Lq, Lk, kv_shared;
+  const int32_t* item_idx;   // optional: shared K/V set of batch item j is item_idx[j] / x_rows
+  int x_rows;
   float scale_log2;
   __nv_bfloat16* o;
   int* err;
@@ -79,7 +82,7 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int bh = blockIdx.y;
   const int head = bh % p.heads, jb = bh / p.heads;
-  const int bkv = p.kv_shared ? head : bh;
+  const int bkv = !p.kv_shared ? bh : (p.item_idx ? (p.item_idx[jb] / p.x_rows) * p.heads + head : head);
   const int q0 = blockIdx.x * 256;
   const int nt = (p.Lk + Cfg::BKV - 1) / Cfg::BKV;
 
@@ -333,9 +336,10 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
 
 template <int HD>
 static cs_status launch_attn(const void* q, const void* k, const void* vt, void* o, int B, int heads, int Lq, int Lk,
-                             int Lkv_stride, int kv_shared, int* err, cudaStream_t stream) {
+                             int Lkv_stride, int kv_shared, int kv_sets, const int32_t* item_idx, int x_rows,
+                             int* err, cudaStream_t stream) {
   using Cfg = AttnCfg<HD>;
-  const int BH = B * heads, Bkv = kv_shared ? heads : BH;
+  const int BH = B * heads, Bkv = kv_shared ? heads * kv_sets : BH;
   CUtensorMap tq, tk, tv;
   {
     const uint64_t dims[3] = {(uint64_t)Cfg::HDS, (uint64_t)Lq, (uint64_t)BH};
@@ -357,6 +361,7 @@ static cs_status launch_attn(const void* q, const void* k, const void* vt, void*
   }
   AttnArgs a{};
   a.B = B; a.heads = heads; a.Lq = Lq; a.Lk = Lk; a.kv_shared = kv_shared;
+  a.item_idx = item_idx; a.x_rows = x_rows > 0 ? x_rows : 1;
   a.scale_log2 = 1.4426950408889634f / sqrtf((float)HD);
   a.o = static_cast<__nv_bfloat16*>(o);
   a.err = err;
@@ -368,19 +373,28 @@ static cs_status launch_attn(const void* q, const void* k, const void* vt, void*
   return CS_OK;
 }
 
-}  // namespace cs
-
-using namespace cs;
-
-extern "C" cs_status cs_attention(const void* q, const void* k, const void* vt, void* o, int B, int heads, int Lq,
-                                  int Lk, int hd, int Lkv_stride, int kv_shared, int* err, cudaStream_t stream) {
+cs_status attention_run(const void* q, const void* k, const void* vt, void* o, int B, int heads, int Lq, int Lk,
+                        int hd, int Lkv_stride, int kv_shared, int kv_sets, const int32_t* item_idx, int x_rows,
+                        int* err, cudaStream_t stream) {
   CS_REQUIRE(q && k && vt && o, "cs_attention: null pointer");
   CS_REQUIRE(B > 0 && heads > 0 && Lq > 0 && Lk > 0, "cs_attention: empty shape");
   CS_REQUIRE(Lkv_stride >= Lk && Lkv_stride % 8 == 0, "cs_attention: Lkv_stride must be >= Lk and a multiple of 8");
   CS_REQUIRE((long long)B * heads <= 65535, "cs_attention: B*heads = %lld exceeds the grid limit",
              (long long)B * heads);
-  if (hd == 128) return launch_attn<128>(q, k, vt, o, B, heads, Lq, Lk, Lkv_stride, kv_shared, err, stream);
-  if (hd == 32) return launch_attn<32>(q, k, vt, o, B, heads, Lq, Lk, Lkv_stride, kv_shared, err, stream);
+  CS_REQUIRE(kv_sets >= 1 && (kv_sets == 1 || (kv_shared && item_idx)), "cs_attention: bad K/V set selection");
+  if (hd == 128)
+    return launch_attn<128>(q, k, vt, o, B, heads, Lq, Lk, Lkv_stride, kv_shared, kv_sets, item_idx, x_rows, err,
+                            stream);
+  if (hd == 32)
+    return launch_attn<32>(q, k, vt, o, B, heads, Lq, Lk, Lkv_stride, kv_shared, kv_sets, item_idx, x_rows, err,
+                           stream);
   set_error("cs_attention: head dim %d not supported (32 or 128)", hd);
   return CS_ERR_UNSUPPORTED;
+}
+
+}  // namespace cs
+
+extern "C" cs_status cs_attention(const void* q, const void* k, const void* vt, void* o, int B, int heads, int Lq,
+                                  int Lk, int hd, int Lkv_stride, int kv_shared, int* err, cudaStream_t stream) {
+  return cs::attention_run(q, k, vt, o, B, heads, Lq, Lk, hd, Lkv_stride, kv_shared, 1, nullptr, 1, err, stream);
 }

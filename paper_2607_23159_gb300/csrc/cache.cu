@@ -61,13 +61,13 @@ __host__ __device__ __forceinline__ bool window_forced(int k, int T, int K_w, in
 // ------------------------------------------------------------------ decide ----
 __global__ void __launch_bounds__(kCacheThreads) drift_partials_kernel(
     const float* __restrict__ x, const float* __restrict__ xr, const uint8_t* __restrict__ has_ref, long long D,
-    int window_forced_step, float* __restrict__ partials) {
+    int window_forced_step, int x_rows, float* __restrict__ partials) {
   const int i = blockIdx.y, c = blockIdx.x, nch = gridDim.x;
   __shared__ float red[2][32];
   if (window_forced_step || !has_ref[i]) return;   // forced step: no drift is evaluated
   const long long lo = (long long)c * kChunkElems;
   const long long hi = min(D, lo + kChunkElems);
-  const float* xi = x + (long long)i * D;
+  const float* xi = x + (long long)(i % x_rows) * D;   // cache state i reads latent row i % x_rows
   const float* ri = xr + (long long)i * D;
   float v[2] = {0.f, 0.f};
   const bool vec = ((D & 3) == 0) && ((reinterpret_cast<uintptr_t>(x) & 15) == 0) &&
@@ -222,6 +222,53 @@ __global__ void __launch_bounds__(kCacheThreads) apply_kernel(float* __restrict_
   }
 }
 
+// Guided update (Eq. cfg with per-branch cache state): state rows i (conditional) and
+// N + i (unconditional) belong to latent row i; each branch's velocity is its DiT output
+// (computed: Delta_b = v_b - x, x_ref_b = x) or x + Delta_b (skipped); the Euler step uses
+// v_u + w (v_c - v_u).
+template <bool kScore>
+__global__ void __launch_bounds__(kCacheThreads) apply_cfg_kernel(
+    float* __restrict__ x, float* __restrict__ xr, float* __restrict__ delta, const float* __restrict__ v,
+    const uint8_t* __restrict__ skip, int N, long long D, float h, float t_next, float w,
+    const float* __restrict__ target, float* __restrict__ partials) {
+  const int i = blockIdx.y, c = blockIdx.x, nch = gridDim.x;
+  __shared__ float red[1][32];
+  const long long lo = (long long)c * kChunkElems;
+  const long long hi = min(D, lo + kChunkElems);
+  const long long xo = (long long)i * D, co = (long long)i * D, uo = (long long)(N + i) * D;
+  const bool sk_c = skip[i] != 0, sk_u = skip[N + i] != 0;
+  float acc[1] = {0.f};
+  for (long long e = lo + threadIdx.x; e < hi; e += kCacheThreads) {
+    const float xv = x[xo + e];
+    float vc, vu;
+    if (sk_c) {
+      vc = xv + delta[co + e];
+    } else {
+      vc = v[co + e];
+      delta[co + e] = vc - xv;
+      xr[co + e] = xv;
+    }
+    if (sk_u) {
+      vu = xv + delta[uo + e];
+    } else {
+      vu = v[uo + e];
+      delta[uo + e] = vu - xv;
+      xr[uo + e] = xv;
+    }
+    const float vg = vu + w * (vc - vu);
+    const float xn = xv + h * vg;
+    x[xo + e] = xn;
+    if (kScore) {
+      const float d0 = xn - t_next * vg - target[e];
+      acc[0] += d0 * d0;
+    }
+  }
+  if (kScore) {
+    block_sum<1>(acc, red);
+    if (threadIdx.x == 0) partials[(long long)i * nch + c] = acc[0];
+  }
+}
+
 // ------------------------------------------------------------------- score ----
 __global__ void __launch_bounds__(kCacheThreads) sqdist_partials_kernel(const float* __restrict__ x,
                                                                         const float* __restrict__ y, long long D,
@@ -329,7 +376,7 @@ extern "C" cs_status cs_cache_decide(const float* x, const float* x_ref, float* 
   const int wf = window_forced(step_k, T, K_w, K_c) ? 1 : 0;
   float* partials = static_cast<float*>(workspace);
   if (!wf) {
-    drift_partials_kernel<<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, has_ref, D, wf, partials);
+    drift_partials_kernel<<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, has_ref, D, wf, N, partials);
     CS_LAUNCHED();
   }
   decide_finalize_kernel<<<1, 256, N, stream>>>(partials, nch, accum, has_ref, N, wf, tau, force, skip_mask, idx,
@@ -356,6 +403,51 @@ extern "C" cs_status cs_cache_apply(float* x, float* x_ref, float* delta, const 
   } else {
     apply_kernel<false><<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, delta, v, skip_mask, D, h, t_next,
                                                                     nullptr, nullptr);
+    CS_LAUNCHED();
+  }
+  return CS_OK;
+}
+
+extern "C" cs_status cs_cache_decide_cfg(const float* x, const float* x_ref, float* accum, uint8_t* has_ref, int N,
+                                         long long D, int step_k, int T, float tau, int K_w, int K_c,
+                                         const uint8_t* force, uint8_t* skip_mask, int32_t* idx,
+                                         int32_t* n_compute, void* workspace, int* err, cudaStream_t stream) {
+  CS_REQUIRE(N > 0 && 2 * N <= 4096 && D > 0, "cs_cache_decide_cfg: need 0 < 2N <= 4096 and D > 0");
+  CS_REQUIRE(x && x_ref && accum && has_ref && skip_mask && idx && n_compute && workspace,
+             "cs_cache_decide_cfg: null pointer");
+  CS_REQUIRE(step_k >= 1 && step_k <= T, "cs_cache_decide_cfg: step %d outside 1..T=%d", step_k, T);
+  const int nch = cache_chunks(D), S = 2 * N;
+  const int wf = window_forced(step_k, T, K_w, K_c) ? 1 : 0;
+  float* partials = static_cast<float*>(workspace);
+  if (!wf) {
+    drift_partials_kernel<<<dim3(nch, S), kCacheThreads, 0, stream>>>(x, x_ref, has_ref, D, wf, N, partials);
+    CS_LAUNCHED();
+  }
+  decide_finalize_kernel<<<1, 256, S, stream>>>(partials, nch, accum, has_ref, S, wf, tau, force, skip_mask, idx,
+                                                n_compute, err);
+  CS_LAUNCHED();
+  return CS_OK;
+}
+
+extern "C" cs_status cs_cache_apply_cfg(float* x, float* x_ref, float* delta, const float* v,
+                                        const uint8_t* skip_mask, int N, long long D, float t_cur, float t_next,
+                                        float w, const float* target, float* scores, void* workspace,
+                                        cudaStream_t stream) {
+  CS_REQUIRE(N > 0 && 2 * N <= 4096 && D > 0, "cs_cache_apply_cfg: need 0 < 2N <= 4096 and D > 0");
+  CS_REQUIRE(x && x_ref && delta && v && skip_mask, "cs_cache_apply_cfg: null pointer");
+  CS_REQUIRE(!target || (scores && workspace), "cs_cache_apply_cfg: scoring needs scores and workspace");
+  const int nch = cache_chunks(D);
+  const float h = t_next - t_cur;
+  float* partials = workspace ? static_cast<float*>(workspace) + (size_t)2 * N * nch * 2 : nullptr;
+  if (target) {
+    apply_cfg_kernel<true><<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, delta, v, skip_mask, N, D, h,
+                                                                       t_next, w, target, partials);
+    CS_LAUNCHED();
+    score_finalize_kernel<<<(N + 127) / 128, 128, 0, stream>>>(partials, nch, N, scores);
+    CS_LAUNCHED();
+  } else {
+    apply_cfg_kernel<false><<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, delta, v, skip_mask, N, D, h,
+                                                                        t_next, w, nullptr, nullptr);
     CS_LAUNCHED();
   }
   return CS_OK;
@@ -458,7 +550,7 @@ extern "C" cs_status cs_cache_decide_noalloc(const float* x, const float* x_ref,
   const int nch = cache_chunks(D);
   const int wf = window_forced(step_k, T, K_w, K_c) ? 1 : 0;
   if (!wf) {
-    drift_partials_kernel<<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, has_ref, D, wf, partials);
+    drift_partials_kernel<<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, has_ref, D, wf, N, partials);
     CS_LAUNCHED();
   }
   decide_finalize_kernel<<<1, 256, N, stream>>>(partials, nch, accum, has_ref, N, wf, tau, force, skip_mask, idx,

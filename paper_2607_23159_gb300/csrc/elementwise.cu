@@ -69,8 +69,8 @@ cs_status layernorm_modulate(const float* x, const float* shift, const float* sc
 // ------------------------------------------------------- patchify / scatter ----
 // tokens[j*L + l][k]: for k < 4C, element (c, f, 2hh+ph, 2ww+pw) of candidate idx[j]
 // with k = 4c + 2ph + pw and l = (f*(H/2) + hh)*(W/2) + ww; columns 4C..Kp-1 are 0.
-__global__ void patchify_kernel(const float* __restrict__ x, const int32_t* __restrict__ idx, int n_c, int C, int F,
-                                int H, int W, int Kp, __nv_bfloat16* __restrict__ tok) {
+__global__ void patchify_kernel(const float* __restrict__ x, const int32_t* __restrict__ idx, int n_c, int x_rows,
+                                int C, int F, int H, int W, int Kp, __nv_bfloat16* __restrict__ tok) {
   const int L = F * (H / 2) * (W / 2);
   const long long total = (long long)n_c * L * Kp;
   const long long D = (long long)C * F * H * W;
@@ -83,7 +83,7 @@ __global__ void patchify_kernel(const float* __restrict__ x, const int32_t* __re
     if (k < 4 * C) {
       const int c = k >> 2, ph = (k >> 1) & 1, pw = k & 1;
       const int ww = l % (W / 2), hh = (l / (W / 2)) % (H / 2), f = l / ((W / 2) * (H / 2));
-      v = x[(long long)idx[j] * D + (((long long)c * F + f) * H + (2 * hh + ph)) * W + (2 * ww + pw)];
+      v = x[(long long)(idx[j] % x_rows) * D + (((long long)c * F + f) * H + (2 * hh + ph)) * W + (2 * ww + pw)];
     }
     tok[t] = __float2bfloat16_rn(v);
   }
@@ -106,11 +106,11 @@ __global__ void unpatchify_kernel(const float* __restrict__ hout, const int32_t*
   }
 }
 
-cs_status patchify(const float* x, const int32_t* idx, int n_c, int C, int F, int H, int W, int Kp,
+cs_status patchify(const float* x, const int32_t* idx, int n_c, int x_rows, int C, int F, int H, int W, int Kp,
                    __nv_bfloat16* tok, cudaStream_t s) {
   const long long total = (long long)n_c * F * (H / 2) * (W / 2) * Kp;
   const int blocks = (int)((total + 255) / 256 < 65535 * 16 ? (total + 255) / 256 : 65535 * 16);
-  patchify_kernel<<<blocks, 256, 0, s>>>(x, idx, n_c, C, F, H, W, Kp, tok);
+  patchify_kernel<<<blocks, 256, 0, s>>>(x, idx, n_c, x_rows, C, F, H, W, Kp, tok);
   CS_LAUNCHED();
   return CS_OK;
 }

@@ -352,3 +352,47 @@ def test_beam_and_pruned_search_degenerate_cases():
     win, sp, ids, _ = O.pruned_search(x1s, T, 0.1, 1, 1, vel, y, prune_step=3, keep=4)
     assert win == i_star
     np.testing.assert_allclose(np.sort(sp), np.sort(sc), rtol=1e-12)
+
+
+def test_cfg_guidance_one_is_conditional_and_tau_zero_is_uncached_guided_sampling():
+    cfg, m = _tiny_model(blocks=1)
+    kv_c = m.text_kv(synth.text_context(cfg))
+    kv_u = m.text_kv(np.zeros((cfg.Lt, cfg.d_text)))
+    vc = lambda x, t: m.velocity(x, t, kv_c)
+    vu = lambda x, t: m.velocity(x, t, kv_u)
+    x1s = synth.initial_noise(cfg, range(2)).astype(np.float64)
+    T = 5
+    # w = 1: the combination is the conditional velocity exactly -> plain conditional sampling
+    sc, su = [O.CacheState() for _ in range(2)], [O.CacheState() for _ in range(2)]
+    xs = x1s
+    for k in range(1, T + 1):
+        xs, _, _, _ = O.search_step_cfg(sc, su, xs, k, T, 0.0, 1, 1, vc, vu, 1.0)
+    for i in range(2):
+        np.testing.assert_allclose(xs[i], O.rollout_uncached(x1s[i], T, vc), rtol=1e-12, atol=1e-12)
+    # w = 0: the unconditional velocity alone
+    sc, su = [O.CacheState() for _ in range(2)], [O.CacheState() for _ in range(2)]
+    xs = x1s
+    for k in range(1, T + 1):
+        xs, _, _, _ = O.search_step_cfg(sc, su, xs, k, T, 0.0, 1, 1, vc, vu, 0.0)
+    for i in range(2):
+        np.testing.assert_allclose(xs[i], O.rollout_uncached(x1s[i], T, vu), rtol=1e-12, atol=1e-12)
+    # w = 5, tau = 0: uncached guided Euler sampling (Eq. cfg + Eq. euler) written out
+    sc, su = [O.CacheState() for _ in range(2)], [O.CacheState() for _ in range(2)]
+    xs = x1s
+    for k in range(1, T + 1):
+        xs, skc, sku, _ = O.search_step_cfg(sc, su, xs, k, T, 0.0, 1, 1, vc, vu, 5.0)
+        assert not skc.any() and not sku.any()
+    t = O.time_grid(T)
+    for i in range(2):
+        x = x1s[i]
+        for k in range(T):
+            a, b = vu(x, t[k]), vc(x, t[k])
+            x = x + (t[k + 1] - t[k]) * (a + 5.0 * (b - a))
+        assert np.array_equal(xs[i], x)
+    # branches keep separate state: with a huge tau each branch skips after its first call
+    sc, su = [O.CacheState()], [O.CacheState()]
+    xs = x1s[:1]
+    for k in range(1, T + 1):
+        xs, skc, sku, _ = O.search_step_cfg(sc, su, xs, k, T, 1e30, 0, 0, vc, vu, 5.0)
+        assert skc[0] == (k > 1) and sku[0] == (k > 1)
+    assert not np.array_equal(sc[0].delta, su[0].delta)
