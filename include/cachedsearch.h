@@ -86,6 +86,15 @@ cs_status cs_destroy_model(cs_model* model);
 cs_status cs_load_weights(cs_model* model, const float* params, size_t count, int params_on_device,
                           cudaStream_t stream);
 
+/* Number of tensors in the parameter layout above (16 + 15 per block). */
+int cs_param_tensor_count(const cs_model_config* cfg);
+
+/* Load one tensor of the layout (index in layout order) from float32 data of exactly its
+ * size, host (params_on_device == 0) or device memory; lets a caller stream a large model
+ * tensor by tensor instead of building the whole flat buffer.  Synchronises the stream. */
+cs_status cs_load_param(cs_model* model, int index, const float* data, size_t count, int params_on_device,
+                        cudaStream_t stream);
+
 /* Project the prompt's text context once per search: ctx_dev [Lt][d_text] float32
  * (device).  Computes text = W2 GELU(W1 ctx + b1) + b2 and each block's
  * cross-attention K/V, cached in the model for every later step (the prompt is shared

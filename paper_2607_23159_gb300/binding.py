@@ -45,6 +45,8 @@ _SIGS = {
     "cs_init_model": (I, [C.POINTER(ModelConfig), C.POINTER(P)]),
     "cs_destroy_model": (I, [P]),
     "cs_load_weights": (I, [P, P, SZ, I, P]),
+    "cs_param_tensor_count": (I, [C.POINTER(ModelConfig)]),
+    "cs_load_param": (I, [P, I, P, SZ, I, P]),
     "cs_set_text_context": (I, [P, P, P]),
     "cs_set_null_text_context": (I, [P, P, P]),
     "cs_dit_forward": (I, [P, P, P, I, F, P, P]),
@@ -224,6 +226,17 @@ class Model:
             flat = np.ascontiguousarray(flat, dtype=np.float32)
         check(lib.cs_load_weights(self.h, _ptr(flat), flat.size if not on_dev else flat.numel(), int(on_dev),
                                   _stream(stream)))
+
+    def load_param(self, index, arr, stream=None):
+        """One tensor of the layout (numpy float32, host)."""
+        arr = np.ascontiguousarray(arr, dtype=np.float32)
+        check(lib.cs_load_param(self.h, index, _ptr(arr), arr.size, 0, _stream(stream)))
+
+    def load_streamed(self, seed=None, threads=None):
+        """Generate the seeded synthetic parameters tensor by tensor and load each."""
+        from . import synth
+        for i, arr in synth.iter_params(self.mcfg, **({} if seed is None else {"seed": seed}), threads=threads):
+            self.load_param(i, arr)
 
     def set_text_context(self, ctx, stream=None):
         check(lib.cs_set_text_context(self.h, _ptr(ctx), _stream(stream)))

@@ -298,65 +298,118 @@ extern "C" cs_status cs_destroy_model(cs_model* m) {
   return CS_OK;
 }
 
+namespace {
+// One parameter tensor of the flat layout: a bf16 GEMM weight (rows x cols, stored with
+// row stride ld) or a float32 vector copied as is.
+struct ParamSlot {
+  bf16* w;
+  float* f;
+  size_t rows, cols, ld;
+  size_t count() const { return w ? rows * cols : rows; }
+};
+
+std::vector<ParamSlot> param_slots(cs_model* m) {
+  const cs_model_config& c = m->cfg;
+  const size_t d = c.d, F = c.ffn, P = m->P;
+  std::vector<ParamSlot> v;
+  auto W = [&](bf16* p, size_t r, size_t cc, size_t ld) { v.push_back({p, nullptr, r, cc, ld}); };
+  auto V = [&](float* p, size_t n) { v.push_back({nullptr, p, n, 1, 1}); };
+  W(m->patch_w, d, P, m->Kp); V(m->patch_b, d);
+  W(m->time_w1, d, c.f_dim, c.f_dim); V(m->time_b1, d);
+  W(m->time_w2, d, d, d); V(m->time_b2, d);
+  W(m->mod_w, 6 * d, d, d); V(m->mod_b, 6 * d);
+  W(m->text_w1, d, c.d_text, c.d_text); V(m->text_b1, d);
+  W(m->text_w2, d, d, d); V(m->text_b2, d);
+  W(m->head_mod_w, 2 * d, d, d); V(m->head_mod_b, 2 * d);
+  W(m->head_w, P, d, d); V(m->head_b, P);
+  for (int b = 0; b < c.blocks; ++b) {
+    BlockW& bw = m->blk[b];
+    V(bw.mod_off, 6 * d);
+    W(bw.qkv_w, 3 * d, d, d); V(bw.qkv_b, 3 * d);
+    W(bw.o_w, d, d, d); V(bw.o_b, d);
+    W(bw.cq_w, d, d, d); V(bw.cq_b, d);
+    W(bw.ckv_w, 2 * d, d, d); V(bw.ckv_b, 2 * d);
+    W(bw.co_w, d, d, d); V(bw.co_b, d);
+    W(bw.ff1_w, F, d, d); V(bw.ff1_b, F);
+    W(bw.ff2_w, d, F, F); V(bw.ff2_b, d);
+  }
+  return v;
+}
+
+// Device float32 source -> destination slot (conversion to bf16 with padding for weights).
+cs_status store_slot(const ParamSlot& sl, const float* src_dev, cudaStream_t s) {
+  if (sl.w) return cs::to_bf16_pad(src_dev, (long long)sl.rows, (int)sl.cols, (int)sl.ld, sl.w, s);
+  CS_CUDA(cudaMemcpyAsync(sl.f, src_dev, sl.rows * sizeof(float), cudaMemcpyDeviceToDevice, s));
+  return CS_OK;
+}
+
+cs_status load_slot(cs_model* m, const ParamSlot& sl, const float* src, int on_device, float* stage,
+                    cudaStream_t s) {
+  if (on_device) return store_slot(sl, src, s);
+  if (!sl.w) {
+    CS_CUDA(cudaMemcpyAsync(sl.f, src, sl.rows * sizeof(float), cudaMemcpyHostToDevice, s));
+    return CS_OK;
+  }
+  CS_CUDA(cudaMemcpyAsync(stage, src, sl.count() * sizeof(float), cudaMemcpyHostToDevice, s));
+  CS_TRY(store_slot(sl, stage, s));
+  CS_CUDA(cudaStreamSynchronize(s));   // the staging buffer is reused by the next tensor
+  (void)m;
+  return CS_OK;
+}
+}  // namespace
+
+extern "C" int cs_param_tensor_count(const cs_model_config* c) {
+  if (!c) return 0;
+  return 16 + 15 * c->blocks;
+}
+
 extern "C" cs_status cs_load_weights(cs_model* m, const float* params, size_t count, int on_device,
                                      cudaStream_t s) {
   CS_REQUIRE(m && params, "cs_load_weights: null pointer");
   const size_t want = cs_param_count(&m->cfg);
   CS_REQUIRE(count == want, "cs_load_weights: got %zu floats, the model has %zu", count, want);
-  const cs_model_config& c = m->cfg;
-  const size_t d = c.d, F = c.ffn, P = m->P;
-  // staging buffer for host input: the largest single tensor
-  size_t biggest = std::max({d * F, 6 * d * d, 3 * d * d, d * (size_t)c.d_text, d * (size_t)c.f_dim});
+  std::vector<ParamSlot> slots = param_slots(m);
+  size_t biggest = 0;
+  for (auto& sl : slots) biggest = std::max(biggest, sl.count());
   float* stage = nullptr;
   if (!on_device) CS_CUDA(cudaMalloc(&stage, biggest * sizeof(float)));
   size_t off = 0;
   cs_status st = CS_OK;
-  auto src_of = [&](size_t n) -> const float* {
-    const float* p = params + off;
-    off += n;
-    if (on_device) return p;
-    if (cudaMemcpyAsync(stage, p, n * sizeof(float), cudaMemcpyHostToDevice, s) != cudaSuccess) st = CS_ERR_CUDA;
-    return stage;
-  };
-  auto w = [&](bf16* dst, size_t rows, size_t cols, size_t ld) {
-    if (st != CS_OK) return;
-    const float* src = src_of(rows * cols);
-    if (st == CS_OK) st = cs::to_bf16_pad(src, (long long)rows, (int)cols, (int)ld, dst, s);
-    if (!on_device && st == CS_OK && cudaStreamSynchronize(s) != cudaSuccess) st = CS_ERR_CUDA;
-  };
-  auto f = [&](float* dst, size_t n) {
-    if (st != CS_OK) return;
-    if (cudaMemcpyAsync(dst, params + off, n * sizeof(float), on_device ? cudaMemcpyDeviceToDevice
-                                                                        : cudaMemcpyHostToDevice, s) != cudaSuccess)
-      st = CS_ERR_CUDA;
-    off += n;
-  };
-  w(m->patch_w, d, P, m->Kp); f(m->patch_b, d);
-  w(m->time_w1, d, c.f_dim, c.f_dim); f(m->time_b1, d);
-  w(m->time_w2, d, d, d); f(m->time_b2, d);
-  w(m->mod_w, 6 * d, d, d); f(m->mod_b, 6 * d);
-  w(m->text_w1, d, c.d_text, c.d_text); f(m->text_b1, d);
-  w(m->text_w2, d, d, d); f(m->text_b2, d);
-  w(m->head_mod_w, 2 * d, d, d); f(m->head_mod_b, 2 * d);
-  w(m->head_w, P, d, d); f(m->head_b, P);
-  for (int b = 0; b < c.blocks; ++b) {
-    BlockW& bw = m->blk[b];
-    f(bw.mod_off, 6 * d);
-    w(bw.qkv_w, 3 * d, d, d); f(bw.qkv_b, 3 * d);
-    w(bw.o_w, d, d, d); f(bw.o_b, d);
-    w(bw.cq_w, d, d, d); f(bw.cq_b, d);
-    w(bw.ckv_w, 2 * d, d, d); f(bw.ckv_b, 2 * d);
-    w(bw.co_w, d, d, d); f(bw.co_b, d);
-    w(bw.ff1_w, F, d, d); f(bw.ff1_b, F);
-    w(bw.ff2_w, d, F, F); f(bw.ff2_b, d);
+  for (auto& sl : slots) {
+    st = load_slot(m, sl, params + off, on_device, stage, s);
+    if (st != CS_OK) break;
+    off += sl.count();
   }
   cudaError_t e = cudaStreamSynchronize(s);
   if (stage) cudaFree(stage);
-  if (st != CS_OK || e != cudaSuccess) {
-    cs::set_error("cs_load_weights: copy or conversion failed (%s)", cudaGetErrorString(e));
+  if (st != CS_OK) return st;
+  if (e != cudaSuccess) {
+    cs::set_error("cs_load_weights: %s", cudaGetErrorString(e));
     return CS_ERR_CUDA;
   }
-  m->text_set = false;
+  m->text_set = m->null_text_set = false;
+  return CS_OK;
+}
+
+extern "C" cs_status cs_load_param(cs_model* m, int index, const float* data, size_t count, int on_device,
+                                   cudaStream_t s) {
+  CS_REQUIRE(m && data, "cs_load_param: null pointer");
+  std::vector<ParamSlot> slots = param_slots(m);
+  CS_REQUIRE(index >= 0 && index < (int)slots.size(), "cs_load_param: tensor index %d outside 0..%d", index,
+             (int)slots.size() - 1);
+  const ParamSlot& sl = slots[index];
+  CS_REQUIRE(count == sl.count(), "cs_load_param: tensor %d has %zu floats, got %zu", index, sl.count(), count);
+  float* stage = nullptr;
+  if (!on_device && sl.w) CS_CUDA(cudaMalloc(&stage, count * sizeof(float)));
+  cs_status st = load_slot(m, sl, data, on_device, stage, s);
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (stage) cudaFree(stage);
+  if (st != CS_OK) return st;
+  if (e != cudaSuccess) {
+    cs::set_error("cs_load_param: %s", cudaGetErrorString(e));
+    return CS_ERR_CUDA;
+  }
+  m->text_set = m->null_text_set = false;
   return CS_OK;
 }
 

@@ -180,6 +180,27 @@ def make_params(m: ModelConfig, seed: int = WEIGHT_SEED, threads: int | None = N
     return flat, views
 
 
+def iter_params(m: ModelConfig, seed: int = WEIGHT_SEED, threads: int | None = None, window: int = 32):
+    """Yield (tensor index, float32 array) in layout order, the same values as
+    :func:`make_params`, generated a bounded window of tensors ahead on a thread pool."""
+    lay = param_layout(m)
+    nthr = threads or min(16, os.cpu_count() or 1)
+
+    def gen(i):
+        name, shape, kind = lay[i]
+        out = np.empty(shape, dtype=np.float32)
+        _one_param(i, shape, kind, seed, out)
+        return out
+
+    with ThreadPoolExecutor(nthr) as ex:
+        futs = {}
+        for i in range(len(lay)):
+            for j in range(i, min(len(lay), i + window)):
+                if j not in futs:
+                    futs[j] = ex.submit(gen, j)
+            yield i, futs.pop(i).result()
+
+
 def normal(seed: int, shape) -> np.ndarray:
     g = np.random.Generator(np.random.Philox(key=seed))
     return g.standard_normal(int(np.prod(shape)), dtype=np.float32).reshape(shape)

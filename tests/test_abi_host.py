@@ -56,3 +56,14 @@ def test_invalid_config_rejected_on_host(b):
     assert "invalid" in b.last_error()
     cfg = b.model_config(synth.replace_model(synth.TINY, heads=2), 4)   # head dim 64
     assert b.lib.cs_init_model(C.byref(cfg), C.byref(h)) == b.CS_ERR_UNSUPPORTED
+
+
+def test_streamed_generator_matches_flat_layout(b):
+    import ctypes as C
+    import numpy as np
+    m = synth.replace_model(synth.TINY, blocks=3)
+    flat, _ = synth.make_params(m)
+    parts = list(synth.iter_params(m, threads=3, window=4))
+    assert [i for i, _ in parts] == list(range(len(parts)))
+    assert len(parts) == b.lib.cs_param_tensor_count(C.byref(b.model_config(m, 1)))
+    assert np.array_equal(np.concatenate([a.reshape(-1) for _, a in parts]), flat)

@@ -240,3 +240,21 @@ def test_wan13b_full_size_properties(B):
     assert float(v4.std()) > 0.05
     assert model.device_error() == 0
     model.close()
+
+
+def test_streamed_weight_loading_equals_flat_loading(B):
+    m = synth.TINY
+    inp = Inputs(m, 2)
+    a = _model(B, inp, 2)
+    b = B.Model(m, 2)
+    b.load_streamed()
+    b.set_text_context(dev(inp.ctx))
+    x = dev(inp.x1.reshape(2, -1))
+    idx = torch.arange(2, dtype=torch.int32, device="cuda")
+    va, vb = torch.zeros(2, m.D, device="cuda"), torch.zeros(2, m.D, device="cuda")
+    a.dit_forward(x, idx, 2, 0.4, va)
+    b.dit_forward(x, idx, 2, 0.4, vb)
+    torch.cuda.synchronize()
+    assert torch.equal(va, vb)
+    a.close()
+    b.close()
