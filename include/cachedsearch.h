@@ -138,9 +138,9 @@ cs_status cs_cache_decide(const float* x_dev, const float* x_ref_dev, float* acc
  * memory: a serving runtime whose memory pool owns the whole device after start-up, or
  * host code that must not let an allocation synchronise the device mid-step.  It takes
  * no workspace; the partial sums live in a fixed array compiled into the library (one
- * per GPU that loads it, kept until the process exits, 64 KB).  The paper has no
+ * per GPU that loads it, kept until the process exits, 256 KB).  The paper has no
  * counterpart: this is a deployment convenience of this library.
- *   Limits: N <= CS_NOALLOC_MAX_N candidates and D <= CS_NOALLOC_MAX_CHUNKS * 32768
+ *   Limits: N <= CS_NOALLOC_MAX_N candidates and D <= CS_NOALLOC_MAX_CHUNKS * 8192
  *   elements per candidate; larger sizes return CS_ERR_ARG with a message, nothing runs.
  *   The first call on a device looks up the array's device address (cudaGetSymbolAddress)
  *   with that device current; make that first call before any stream capture.
@@ -149,7 +149,7 @@ cs_status cs_cache_decide(const float* x_dev, const float* x_ref_dev, float* acc
  *   partial it reads, so nothing from a previous call needs clearing.
  * Arguments, results and errors are those of cs_cache_decide. */
 #define CS_NOALLOC_MAX_N 64
-#define CS_NOALLOC_MAX_CHUNKS 128
+#define CS_NOALLOC_MAX_CHUNKS 512
 cs_status cs_cache_decide_noalloc(const float* x_dev, const float* x_ref_dev, float* accum_dev,
                                   uint8_t* has_ref_dev, int N, long long D, int step_k, int T, float tau,
                                   int K_w, int K_c, const uint8_t* force_compute_dev, uint8_t* skip_mask_dev,
@@ -191,8 +191,28 @@ cs_status cs_search_step_cfg(cs_model* model, float* x_dev, float* x_ref_dev, fl
                              uint8_t* skip_mask_dev, const float* target_dev, float* scores_dev, int* n_computed,
                              cudaStream_t stream);
 
+/* Single-pass form used by cs_search_step.  cs_cache_decide_skip takes the decision of
+ * every candidate (as cs_cache_decide) and, in the same launch, applies Eq. skip + Eq.
+ * euler to the skipped ones (and writes their score partials if target_dev is given), so
+ * a skipped candidate's x, x_ref and Delta are read once and x written once.  One
+ * cooperative launch with a bounded grid barrier; needs D % 4 == 0, 16-byte aligned
+ * tensors and cs_cache_workspace_bytes(N, D) of workspace (its barrier words are reset
+ * by the call).  cs_cache_apply_computed then updates only the computed candidates
+ * (Eq. delta + Eq. euler, v_dev from the DiT) and, with target_dev, finalises the scores
+ * of all candidates. */
+cs_status cs_cache_decide_skip(float* x_dev, const float* x_ref_dev, const float* delta_dev, float* accum_dev,
+                               uint8_t* has_ref_dev, int N, long long D, int step_k, int T, float t_cur,
+                               float t_next, float tau, int K_w, int K_c, const uint8_t* force_compute_dev,
+                               uint8_t* skip_mask_dev, int32_t* compute_idx_dev, int32_t* n_compute_dev,
+                               const float* target_dev, void* workspace_dev, int* err_dev, cudaStream_t stream);
+cs_status cs_cache_apply_computed(float* x_dev, float* x_ref_dev, float* delta_dev, const float* v_dev,
+                                  const uint8_t* skip_mask_dev, int N, long long D, float t_cur, float t_next,
+                                  const float* target_dev, float* scores_dev, void* workspace_dev,
+                                  cudaStream_t stream);
+
 /* One denoising step of N candidates (the unit of work of the search):
- * cs_cache_decide, then cs_dit_forward on the computing subset, then cs_cache_apply.
+ * cs_cache_decide_skip, then cs_dit_forward on the computing subset, then
+ * cs_cache_apply_computed.
  * State buffers (x, x_ref, delta: [N][D]; accum: [N]; has_ref: [N]) are caller-owned
  * device memory and are updated in place; a fresh search starts with has_ref = 0.
  * Synchronises once to read the number of computing candidates; that count is returned

@@ -57,6 +57,8 @@ _SIGS = {
     "cs_cache_decide": (I, [P, P, P, P, I, LL, I, I, F, I, I, P, P, P, P, P, P, P]),
     "cs_cache_decide_noalloc": (I, [P, P, P, P, I, LL, I, I, F, I, I, P, P, P, P, P, P]),
     "cs_cache_apply": (I, [P, P, P, P, P, I, LL, F, F, P, P, P, P]),
+    "cs_cache_decide_skip": (I, [P, P, P, P, P, I, LL, I, I, F, F, F, I, I, P, P, P, P, P, P, P, P]),
+    "cs_cache_apply_computed": (I, [P, P, P, P, P, I, LL, F, F, P, P, P, P]),
     "cs_search_step": (I, [P, P, P, P, P, P, I, I, I, F, F, F, I, I, P, P, P, P, P, P]),
     "cs_search_step_host": (I, [P, P, P, P, P, P, I, I, I, F, F, F, I, I, P, P, P]),
     "cs_score": (I, [P, P, I, LL, P, P, P]),
@@ -174,6 +176,23 @@ def cache_apply(x, x_ref, delta, v, skip_mask, t_cur, t_next, workspace=None, ta
     Dn = x[0].numel()
     check(lib.cs_cache_apply(_ptr(x), _ptr(x_ref), _ptr(delta), _ptr(v), _ptr(skip_mask), N, Dn, t_cur, t_next,
                              _ptr(target), _ptr(scores), _ptr(workspace), _stream(stream)))
+
+
+def cache_decide_skip(x, x_ref, delta, accum, has_ref, step_k, T, t_cur, t_next, tau, K_w, K_c, skip_mask,
+                      compute_idx, n_compute, workspace, force=None, target=None, err=None, stream=None):
+    N = x.shape[0]
+    check(lib.cs_cache_decide_skip(_ptr(x), _ptr(x_ref), _ptr(delta), _ptr(accum), _ptr(has_ref), N, x[0].numel(),
+                                   step_k, T, t_cur, t_next, tau, K_w, K_c, _ptr(force), _ptr(skip_mask),
+                                   _ptr(compute_idx), _ptr(n_compute), _ptr(target), _ptr(workspace), _ptr(err),
+                                   _stream(stream)))
+
+
+def cache_apply_computed(x, x_ref, delta, v, skip_mask, t_cur, t_next, workspace=None, target=None, scores=None,
+                         stream=None):
+    N = x.shape[0]
+    check(lib.cs_cache_apply_computed(_ptr(x), _ptr(x_ref), _ptr(delta), _ptr(v), _ptr(skip_mask), N,
+                                      x[0].numel(), t_cur, t_next, _ptr(target), _ptr(scores), _ptr(workspace),
+                                      _stream(stream)))
 
 
 def score(x, target, scores, workspace, stream=None):

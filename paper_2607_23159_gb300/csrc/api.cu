@@ -517,8 +517,9 @@ static cs_status step_impl(cs_model* m, float* x, float* x_ref, float* delta, fl
   cudaEvent_t ev[2];
   const bool wf = k <= K_w || k > T - K_c;
   CS_TRY(record_begin(m, 3, s, ev));
-  CS_TRY(cs_cache_decide(x, x_ref, accum, has_ref, N, D, k, T, tau, K_w, K_c, force, skip, m->idx, m->n_compute,
-                         m->cache_ws, m->err, s));
+  // decision + the update of skipped candidates in one pass; computed ones after the DiT
+  CS_TRY(cs_cache_decide_skip(x, x_ref, delta, accum, has_ref, N, D, k, T, t_cur, t_next, tau, K_w, K_c, force, skip,
+                              m->idx, m->n_compute, target, m->cache_ws, m->err, s));
   CS_TRY(record_end(m, 3, s, ev, 0.0));
   CS_CUDA(cudaMemcpyAsync(m->n_host, m->n_compute, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
   CS_CUDA(cudaMemcpyAsync(m->n_host + 1, m->err, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
@@ -533,7 +534,8 @@ static cs_status step_impl(cs_model* m, float* x, float* x_ref, float* delta, fl
   if (n_out) *n_out = n_c;
   CS_TRY(dit_forward_impl(m, x, m->idx, n_c, N, 1, t_cur, m->v, s));
   CS_TRY(record_begin(m, 3, s, ev));
-  CS_TRY(cs_cache_apply(x, x_ref, delta, m->v, skip, N, D, t_cur, t_next, target, scores, m->cache_ws, s));
+  if (n_c > 0 || target)
+    CS_TRY(cs_cache_apply_computed(x, x_ref, delta, m->v, skip, N, D, t_cur, t_next, target, scores, m->cache_ws, s));
   // algorithmic bytes of indicator + update (each tensor read or written once):
   //   skipped: read x, x_ref, Delta, write x                       16 D
   //   computed: read x, v (+ x_ref on a free step), write x, Delta, x_ref   20 D (24 D)

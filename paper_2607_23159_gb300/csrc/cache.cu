@@ -21,7 +21,7 @@
 namespace cs {
 
 constexpr int kCacheThreads = 256;
-constexpr long long kChunkElems = 32768;   // elements of one candidate per CTA (multiple of 4*256)
+constexpr long long kChunkElems = 8192;    // elements of one candidate per CTA (multiple of 4*256)
 
 __host__ __device__ inline int cache_chunks(long long D) {
   long long c = (D + kChunkElems - 1) / kChunkElems;
@@ -54,6 +54,34 @@ __device__ __forceinline__ void block_sum(float (&v)[NV], float (*red)[32]) {
   }
 }
 
+// 256-bit global loads with an L2 eviction-priority hint: data read again soon (x, re-read
+// by the update after the decision) is kept, data used once is dropped first.
+struct F8 {
+  float v[8];
+};
+#define CS_LD8(QUAL)                                                                                      \
+  asm volatile("ld.global.L1::no_allocate.L2::" QUAL ".v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];" \
+               : "=r"(u[0]), "=r"(u[1]), "=r"(u[2]), "=r"(u[3]), "=r"(u[4]), "=r"(u[5]), "=r"(u[6]),      \
+                 "=r"(u[7])                                                                               \
+               : "l"(p))
+__device__ __forceinline__ F8 ld8_keep(const float* p) {
+  uint32_t u[8];
+  CS_LD8("evict_last");
+  F8 r;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) r.v[j] = __uint_as_float(u[j]);
+  return r;
+}
+__device__ __forceinline__ F8 ld8_once(const float* p) {
+  uint32_t u[8];
+  CS_LD8("evict_first");
+  F8 r;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) r.v[j] = __uint_as_float(u[j]);
+  return r;
+}
+#undef CS_LD8
+
 __host__ __device__ __forceinline__ bool window_forced(int k, int T, int K_w, int K_c) {
   return k <= K_w || k > T - K_c;
 }
@@ -70,18 +98,19 @@ __global__ void __launch_bounds__(kCacheThreads) drift_partials_kernel(
   const float* xi = x + (long long)(i % x_rows) * D;   // cache state i reads latent row i % x_rows
   const float* ri = xr + (long long)i * D;
   float v[2] = {0.f, 0.f};
-  const bool vec = ((D & 3) == 0) && ((reinterpret_cast<uintptr_t>(x) & 15) == 0) &&
-                   ((reinterpret_cast<uintptr_t>(xr) & 15) == 0);
+  const bool vec = ((D & 7) == 0) && ((reinterpret_cast<uintptr_t>(x) & 31) == 0) &&
+                   ((reinterpret_cast<uintptr_t>(xr) & 31) == 0);
   if (vec) {
-    const float4* x4 = reinterpret_cast<const float4*>(xi + lo);
-    const float4* r4 = reinterpret_cast<const float4*>(ri + lo);
-    const int n4 = (int)((hi - lo) >> 2);
+    const int n8 = (int)((hi - lo) >> 3);
 #pragma unroll 4
-    for (int e = threadIdx.x; e < n4; e += kCacheThreads) {
-      const float4 a = __ldcs(x4 + e), b = __ldcs(r4 + e);
-      const float d0 = a.x - b.x, d1 = a.y - b.y, d2 = a.z - b.z, d3 = a.w - b.w;
-      v[0] += d0 * d0 + d1 * d1 + d2 * d2 + d3 * d3;
-      v[1] += b.x * b.x + b.y * b.y + b.z * b.z + b.w * b.w;
+    for (int e = threadIdx.x; e < n8; e += kCacheThreads) {
+      const F8 a = ld8_keep(xi + lo + 8 * e), b = ld8_once(ri + lo + 8 * e);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float dd = a.v[j] - b.v[j];
+        v[0] += dd * dd;
+        v[1] += b.v[j] * b.v[j];
+      }
     }
   } else {
     for (long long e = lo + threadIdx.x; e < hi; e += kCacheThreads) {
@@ -97,47 +126,63 @@ __global__ void __launch_bounds__(kCacheThreads) drift_partials_kernel(
   }
 }
 
+// Fixed-order sum of one candidate's chunk partials by one warp: lane l takes chunks
+// l, l+32, ... in order, then a fixed shuffle tree (the order depends only on nch).
+__device__ __forceinline__ double warp_sum_partials(const float* __restrict__ p, int nch, int stride, int lane) {
+  double s = 0.0;
+  for (int c = lane; c < nch; c += 32) s += (double)p[(long long)c * stride];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  return s;
+}
+
+// One warp per candidate: drift from the partials, accumulate, decide; then thread 0
+// writes the ordered compaction list.
 __global__ void decide_finalize_kernel(const float* __restrict__ partials, int nch, float* __restrict__ accum,
                                        uint8_t* __restrict__ has_ref, int N, int window_forced_step, float tau,
                                        const uint8_t* __restrict__ force, uint8_t* __restrict__ skip_mask,
                                        int32_t* __restrict__ idx, int32_t* __restrict__ n_compute, int* err) {
   extern __shared__ uint8_t flags[];
-  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  for (int i = warp; i < N; i += nw) {
     const bool had = has_ref[i] != 0;
-    bool compute;
-    float a = accum[i];
-    if (window_forced_step || !had) {
-      compute = true;
-    } else {
-      double num = 0.0, den = 0.0;
-      for (int c = 0; c < nch; ++c) {
-        num += (double)partials[((long long)i * nch + c) * 2 + 0];
-        den += (double)partials[((long long)i * nch + c) * 2 + 1];
-      }
-      const double drift = sqrt(num) / sqrt(den);
-      if (!isfinite(drift)) {
-        record_error(err, CS_ERR_NONFINITE);
+    const bool free_step = !window_forced_step && had;
+    double num = 0.0, den = 0.0;
+    if (free_step) {
+      num = warp_sum_partials(partials + (long long)i * nch * 2 + 0, nch, 2, lane);
+      den = warp_sum_partials(partials + (long long)i * nch * 2 + 1, nch, 2, lane);
+    }
+    if (lane == 0) {
+      bool compute;
+      float a = accum[i];
+      if (!free_step) {
         compute = true;
       } else {
-        a = (float)((double)a + drift);
-        compute = (tau <= 0.f) || (a > tau);
+        const double drift = sqrt(num) / sqrt(den);
+        if (!isfinite(drift)) {
+          record_error(err, CS_ERR_NONFINITE);
+          compute = true;
+        } else {
+          a = (float)((double)a + drift);
+          compute = (tau <= 0.f) || (a > tau);
+        }
       }
-    }
-    if (force) {
-      const bool f = force[i] != 0;
-      if (!f && !had) {
-        record_error(err, CS_ERR_ARG);
-      } else {
-        compute = f;
+      if (force) {
+        const bool f = force[i] != 0;
+        if (!f && !had) {
+          record_error(err, CS_ERR_ARG);
+        } else {
+          compute = f;
+        }
       }
+      if (compute) {
+        a = 0.f;
+        has_ref[i] = 1;
+      }
+      accum[i] = a;
+      skip_mask[i] = compute ? 0 : 1;
+      flags[i] = compute ? 1 : 0;
     }
-    if (compute) {
-      a = 0.f;
-      has_ref[i] = 1;
-    }
-    accum[i] = a;
-    skip_mask[i] = compute ? 0 : 1;
-    flags[i] = compute ? 1 : 0;
   }
   __syncthreads();
   if (threadIdx.x == 0) {
@@ -176,7 +221,7 @@ __global__ void __launch_bounds__(kCacheThreads) apply_kernel(float* __restrict_
     const float4* v4 = reinterpret_cast<const float4*>(v + base + lo);
     const float4* y4 = reinterpret_cast<const float4*>(target + lo);
     const int n4 = (int)((hi - lo) >> 2);
-#pragma unroll 2
+#pragma unroll 4
     for (int e = threadIdx.x; e < n4; e += kCacheThreads) {
       const float4 xv = __ldcs(x4 + e);
       float4 vu, xn;
@@ -302,10 +347,225 @@ __global__ void __launch_bounds__(kCacheThreads) sqdist_partials_kernel(const fl
 
 __global__ void score_finalize_kernel(const float* __restrict__ partials, int nch, int N,
                                       float* __restrict__ scores) {
-  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < N; i += gridDim.x * blockDim.x) {
-    double s = 0.0;
-    for (int c = 0; c < nch; ++c) s += (double)partials[(long long)i * nch + c];
-    scores[i] = (float)(-sqrt(s));
+  const int lane = threadIdx.x & 31;
+  const int w0 = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, nw = (gridDim.x * blockDim.x) >> 5;
+  for (int i = w0; i < N; i += nw) {
+    const double s = warp_sum_partials(partials + (long long)i * nch, nch, 1, lane);
+    if (lane == 0) scores[i] = (float)(-sqrt(s));
+  }
+}
+
+// ---------------------------------------------------- fused decide + skip ----
+// One cooperative launch per step: (1) drift partials of every (candidate, chunk) on a
+// free step, (2) a grid barrier, (3) every CTA derives all decisions from the partials
+// (the same fixed-order sums everywhere), CTA 0 stores the state and compaction list,
+// (4) skipped candidates get Eq. skip + Eq. euler (and their x0-score partials) while
+// computed ones wait for the DiT.  Phase (4) walks the chunks in reverse so the x just
+// read in phase (1) is still in L2.
+
+// Grid-wide barrier over co-resident CTAs (cooperative launch), bounded in time.
+// bar[0] counts arrivals, bar[1] is the generation; bar[0] must be 0 at launch.
+__device__ __forceinline__ void grid_barrier(unsigned* bar, int* err) {
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    volatile unsigned* gen = bar + 1;
+    const unsigned g = *gen;
+    __threadfence();
+    if (atomicAdd(bar, 1u) == gridDim.x - 1) {
+      atomicExch(bar, 0u);
+      __threadfence();
+      atomicAdd(bar + 1, 1u);
+    } else {
+      const uint64_t t0 = globaltimer_ns();
+      while (*gen == g) {
+        __nanosleep(64);
+        if (globaltimer_ns() - t0 > CS_WAIT_TIMEOUT_NS) {
+          record_error(err, kErrTimeout);
+          break;
+        }
+      }
+    }
+    __threadfence();
+  }
+  __syncthreads();
+}
+
+template <bool kScore>
+__global__ void __launch_bounds__(kCacheThreads) decide_skip_kernel(
+    float* __restrict__ x, const float* __restrict__ xr, const float* __restrict__ delta, float* __restrict__ accum,
+    uint8_t* __restrict__ has_ref, int N, long long D, int nch, int wf, float tau, const uint8_t* __restrict__ force,
+    uint8_t* __restrict__ skip_mask, int32_t* __restrict__ idx, int32_t* __restrict__ n_compute, float h,
+    float t_next, const float* __restrict__ target, float* __restrict__ partials, float* __restrict__ spart,
+    unsigned* bar, int* err) {
+  __shared__ float red[2][32];
+  extern __shared__ float sm_dyn[];
+  float* a_s = sm_dyn;                                      // [N] accumulator before this step
+  uint8_t* had = reinterpret_cast<uint8_t*>(a_s + N);       // [N] has_ref before this step
+  uint8_t* dec = had + N;                                   // [N] 1 = compute, 0 = skip
+  const int items = N * nch;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  // this CTA's contiguous range of (candidate, chunk) items
+  const int per = (items + gridDim.x - 1) / gridDim.x;
+  const int it0 = blockIdx.x * per, it1 = min(items, it0 + per);
+  // (0) snapshot the per-candidate state: CTA 0 rewrites it after the barrier
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    a_s[i] = accum[i];
+    had[i] = has_ref[i];
+  }
+  __syncthreads();
+  // (1) drift partials
+  if (!wf) {
+    for (int item = it0; item < it1; ++item) {
+      const int i = item / nch, c = item % nch;
+      if (!had[i]) continue;
+      const long long lo = (long long)c * kChunkElems, hi = min(D, lo + kChunkElems);
+      const float* xi = x + (long long)i * D + lo;
+      const float* ri = xr + (long long)i * D + lo;
+      const int n8 = (int)((hi - lo) >> 3);
+      float v[2] = {0.f, 0.f};
+#pragma unroll 4
+      for (int e = threadIdx.x; e < n8; e += kCacheThreads) {
+        const F8 a = ld8_keep(xi + 8 * e), b = ld8_once(ri + 8 * e);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float dd = a.v[j] - b.v[j];
+          v[0] += dd * dd;
+          v[1] += b.v[j] * b.v[j];
+        }
+      }
+      block_sum<2>(v, red);
+      if (threadIdx.x == 0) {
+        partials[((long long)i * nch + c) * 2 + 0] = v[0];
+        partials[((long long)i * nch + c) * 2 + 1] = v[1];
+      }
+      __syncthreads();
+    }
+  }
+  // (2) every partial is written
+  grid_barrier(bar, err);
+  // (3) decisions (the same fixed-order sums in every CTA): CTA 0 takes every candidate
+  // and stores the state, the others only the candidates of their own range
+  const int c_lo = blockIdx.x == 0 ? 0 : (it0 < it1 ? it0 / nch : 0);
+  const int c_hi = blockIdx.x == 0 ? N : (it0 < it1 ? (it1 - 1) / nch + 1 : 0);
+  for (int i = c_lo + warp; i < c_hi; i += nw) {
+    const bool hr = had[i] != 0;
+    const bool free_step = !wf && hr;
+    double num = 0.0, den = 0.0;
+    if (free_step) {
+      num = warp_sum_partials(partials + (long long)i * nch * 2 + 0, nch, 2, lane);
+      den = warp_sum_partials(partials + (long long)i * nch * 2 + 1, nch, 2, lane);
+    }
+    if (lane == 0) {
+      bool compute = true;
+      float a = a_s[i];
+      if (free_step) {
+        const double drift = sqrt(num) / sqrt(den);
+        if (!isfinite(drift)) {
+          if (blockIdx.x == 0) record_error(err, CS_ERR_NONFINITE);
+        } else {
+          a = (float)((double)a + drift);
+          compute = (tau <= 0.f) || (a > tau);
+        }
+      }
+      if (force) {
+        const bool f = force[i] != 0;
+        if (!f && !hr) {
+          if (blockIdx.x == 0) record_error(err, CS_ERR_ARG);
+        } else {
+          compute = f;
+        }
+      }
+      dec[i] = compute ? 1 : 0;
+      if (blockIdx.x == 0) {
+        accum[i] = compute ? 0.f : a;
+        skip_mask[i] = compute ? 0 : 1;
+      }
+    }
+  }
+  __syncthreads();
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    int n = 0;
+    for (int i = 0; i < N; ++i)
+      if (dec[i]) {
+        idx[n++] = i;
+        has_ref[i] = 1;
+      }
+    *n_compute = n;
+  }
+  // (4) skipped candidates of this range: x += h (x + Delta), newest chunks first
+  for (int item = it1 - 1; item >= it0; --item) {
+    const int i = item / nch, c = item % nch;
+    if (dec[i]) continue;
+    const long long lo = (long long)c * kChunkElems, hi = min(D, lo + kChunkElems);
+    float* xi = x + (long long)i * D + lo;
+    const float* di = delta + (long long)i * D + lo;
+    const float* yi = kScore ? target + lo : nullptr;
+    const int n8 = (int)((hi - lo) >> 3);
+    float acc[1] = {0.f};
+#pragma unroll 2
+    for (int e = threadIdx.x; e < n8; e += kCacheThreads) {
+      const F8 xv = ld8_once(xi + 8 * e), dv = ld8_once(di + 8 * e);
+      float xn[8], vu[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        vu[j] = xv.v[j] + dv.v[j];              // Eq. skip
+        xn[j] = xv.v[j] + h * vu[j];            // Eq. euler
+      }
+      float4* o4 = reinterpret_cast<float4*>(xi + 8 * e);
+      __stcs(o4, make_float4(xn[0], xn[1], xn[2], xn[3]));
+      __stcs(o4 + 1, make_float4(xn[4], xn[5], xn[6], xn[7]));
+      if (kScore) {
+        const F8 y = ld8_once(yi + 8 * e);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float d0 = xn[j] - t_next * vu[j] - y.v[j];
+          acc[0] += d0 * d0;
+        }
+      }
+    }
+    if (kScore) {
+      block_sum<1>(acc, red);
+      if (threadIdx.x == 0) spart[(long long)i * nch + c] = acc[0];
+      __syncthreads();
+    }
+  }
+}
+
+// The update of computed candidates only (skipped ones were updated by decide_skip).
+template <bool kScore>
+__global__ void __launch_bounds__(kCacheThreads) apply_computed_kernel(
+    float* __restrict__ x, float* __restrict__ xr, float* __restrict__ delta, const float* __restrict__ v,
+    const uint8_t* __restrict__ skip, long long D, float h, float t_next, const float* __restrict__ target,
+    float* __restrict__ spart) {
+  const int i = blockIdx.y, c = blockIdx.x, nch = gridDim.x;
+  if (skip[i]) return;
+  __shared__ float red[1][32];
+  const long long lo = (long long)c * kChunkElems, hi = min(D, lo + kChunkElems);
+  const long long base = (long long)i * D;
+  float4* x4 = reinterpret_cast<float4*>(x + base + lo);
+  float4* r4 = reinterpret_cast<float4*>(xr + base + lo);
+  float4* d4 = reinterpret_cast<float4*>(delta + base + lo);
+  const float4* v4 = reinterpret_cast<const float4*>(v + base + lo);
+  const float4* y4 = kScore ? reinterpret_cast<const float4*>(target + lo) : nullptr;
+  const int n4 = (int)((hi - lo) >> 2);
+  float acc[1] = {0.f};
+#pragma unroll 4
+  for (int e = threadIdx.x; e < n4; e += kCacheThreads) {
+    const float4 xv = __ldcs(x4 + e), vu = __ldcs(v4 + e);
+    __stcs(d4 + e, make_float4(vu.x - xv.x, vu.y - xv.y, vu.z - xv.z, vu.w - xv.w));
+    __stcs(r4 + e, xv);
+    const float4 xn = make_float4(xv.x + h * vu.x, xv.y + h * vu.y, xv.z + h * vu.z, xv.w + h * vu.w);
+    __stcs(x4 + e, xn);
+    if (kScore) {
+      const float4 y = __ldg(y4 + e);
+      const float e0 = xn.x - t_next * vu.x - y.x, e1 = xn.y - t_next * vu.y - y.y;
+      const float e2 = xn.z - t_next * vu.z - y.z, e3 = xn.w - t_next * vu.w - y.w;
+      acc[0] += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
+    }
+  }
+  if (kScore) {
+    block_sum<1>(acc, red);
+    if (threadIdx.x == 0) spart[(long long)i * nch + c] = acc[0];
   }
 }
 
@@ -361,7 +621,7 @@ using namespace cs;
 
 extern "C" size_t cs_cache_workspace_bytes(int N, long long D) {
   if (N <= 0 || D <= 0) return 0;
-  return (size_t)N * (size_t)cache_chunks(D) * 3 * sizeof(float);
+  return (size_t)N * (size_t)cache_chunks(D) * 3 * sizeof(float) + 256;   // + grid-barrier words
 }
 
 extern "C" cs_status cs_cache_decide(const float* x, const float* x_ref, float* accum, uint8_t* has_ref, int N,
@@ -379,7 +639,7 @@ extern "C" cs_status cs_cache_decide(const float* x, const float* x_ref, float* 
     drift_partials_kernel<<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, has_ref, D, wf, N, partials);
     CS_LAUNCHED();
   }
-  decide_finalize_kernel<<<1, 256, N, stream>>>(partials, nch, accum, has_ref, N, wf, tau, force, skip_mask, idx,
+  decide_finalize_kernel<<<1, 1024, N, stream>>>(partials, nch, accum, has_ref, N, wf, tau, force, skip_mask, idx,
                                                 n_compute, err);
   CS_LAUNCHED();
   return CS_OK;
@@ -398,7 +658,7 @@ extern "C" cs_status cs_cache_apply(float* x, float* x_ref, float* delta, const 
     apply_kernel<true><<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, delta, v, skip_mask, D, h, t_next,
                                                                    target, partials);
     CS_LAUNCHED();
-    score_finalize_kernel<<<(N + 127) / 128, 128, 0, stream>>>(partials, nch, N, scores);
+    score_finalize_kernel<<<(N + 3) / 4, 128, 0, stream>>>(partials, nch, N, scores);
     CS_LAUNCHED();
   } else {
     apply_kernel<false><<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, delta, v, skip_mask, D, h, t_next,
@@ -423,7 +683,7 @@ extern "C" cs_status cs_cache_decide_cfg(const float* x, const float* x_ref, flo
     drift_partials_kernel<<<dim3(nch, S), kCacheThreads, 0, stream>>>(x, x_ref, has_ref, D, wf, N, partials);
     CS_LAUNCHED();
   }
-  decide_finalize_kernel<<<1, 256, S, stream>>>(partials, nch, accum, has_ref, S, wf, tau, force, skip_mask, idx,
+  decide_finalize_kernel<<<1, 1024, S, stream>>>(partials, nch, accum, has_ref, S, wf, tau, force, skip_mask, idx,
                                                 n_compute, err);
   CS_LAUNCHED();
   return CS_OK;
@@ -443,11 +703,78 @@ extern "C" cs_status cs_cache_apply_cfg(float* x, float* x_ref, float* delta, co
     apply_cfg_kernel<true><<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, delta, v, skip_mask, N, D, h,
                                                                        t_next, w, target, partials);
     CS_LAUNCHED();
-    score_finalize_kernel<<<(N + 127) / 128, 128, 0, stream>>>(partials, nch, N, scores);
+    score_finalize_kernel<<<(N + 3) / 4, 128, 0, stream>>>(partials, nch, N, scores);
     CS_LAUNCHED();
   } else {
     apply_cfg_kernel<false><<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, delta, v, skip_mask, N, D, h,
                                                                         t_next, w, nullptr, nullptr);
+    CS_LAUNCHED();
+  }
+  return CS_OK;
+}
+
+// Bytes past cs_cache_workspace_bytes used by the fused pair: the grid-barrier words.
+static size_t barrier_offset(int N, long long D) { return (size_t)N * cache_chunks(D) * 3 * sizeof(float); }
+
+extern "C" cs_status cs_cache_decide_skip(float* x, const float* x_ref, const float* delta, float* accum,
+                                          uint8_t* has_ref, int N, long long D, int step_k, int T, float t_cur,
+                                          float t_next, float tau, int K_w, int K_c, const uint8_t* force,
+                                          uint8_t* skip_mask, int32_t* idx, int32_t* n_compute,
+                                          const float* target, void* workspace, int* err, cudaStream_t stream) {
+  CS_REQUIRE(N > 0 && N <= 4096 && D > 0, "cs_cache_decide_skip: need 0 < N <= 4096 and D > 0");
+  CS_REQUIRE(x && x_ref && delta && accum && has_ref && skip_mask && idx && n_compute && workspace,
+             "cs_cache_decide_skip: null pointer");
+  CS_REQUIRE(step_k >= 1 && step_k <= T, "cs_cache_decide_skip: step %d outside 1..T=%d", step_k, T);
+  CS_REQUIRE((D & 7) == 0 && (reinterpret_cast<uintptr_t>(x) & 31) == 0 &&
+                 (reinterpret_cast<uintptr_t>(x_ref) & 31) == 0 && (reinterpret_cast<uintptr_t>(delta) & 31) == 0 &&
+                 (!target || (reinterpret_cast<uintptr_t>(target) & 31) == 0),
+             "cs_cache_decide_skip: needs D %% 8 == 0 and 32-byte aligned tensors");
+  const int nch = cache_chunks(D);
+  int wf = window_forced(step_k, T, K_w, K_c) ? 1 : 0;
+  float* partials = static_cast<float*>(workspace);
+  float* spart = partials + (size_t)N * nch * 2;
+  unsigned* bar = reinterpret_cast<unsigned*>(static_cast<char*>(workspace) + barrier_offset(N, D));
+  CS_CUDA(cudaMemsetAsync(bar, 0, 2 * sizeof(unsigned), stream));
+  float h = t_next - t_cur;
+  const bool score = target != nullptr;
+  void* kern = score ? (void*)decide_skip_kernel<true> : (void*)decide_skip_kernel<false>;
+  int per_sm = 0;
+  const size_t dyn = (size_t)N * 6;
+  CS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kCacheThreads, dyn));
+  if (per_sm < 1) {
+    set_error("cs_cache_decide_skip: kernel does not fit on an SM");
+    return CS_ERR_CUDA;
+  }
+  int grid = num_sms() * (per_sm < 8 ? per_sm : 8);
+  const int items = N * nch;
+  if (grid > items) grid = items;
+  void* args[] = {&x, (void*)&x_ref, (void*)&delta, &accum, &has_ref, &N, &D, (void*)&nch, &wf, &tau,
+                  (void*)&force, &skip_mask, &idx, &n_compute, &h, &t_next, (void*)&target, &partials, &spart, &bar,
+                  &err};
+  CS_CUDA(cudaLaunchCooperativeKernel(kern, dim3(grid), dim3(kCacheThreads), args, dyn, stream));
+  count_launch();
+  return CS_OK;
+}
+
+extern "C" cs_status cs_cache_apply_computed(float* x, float* x_ref, float* delta, const float* v,
+                                             const uint8_t* skip_mask, int N, long long D, float t_cur, float t_next,
+                                             const float* target, float* scores, void* workspace,
+                                             cudaStream_t stream) {
+  CS_REQUIRE(N > 0 && N <= 4096 && D > 0 && (D & 3) == 0, "cs_cache_apply_computed: bad sizes");
+  CS_REQUIRE(x && x_ref && delta && v && skip_mask, "cs_cache_apply_computed: null pointer");
+  CS_REQUIRE(!target || (scores && workspace), "cs_cache_apply_computed: scoring needs scores and workspace");
+  const int nch = cache_chunks(D);
+  const float h = t_next - t_cur;
+  float* spart = workspace ? static_cast<float*>(workspace) + (size_t)N * nch * 2 : nullptr;
+  if (target) {
+    apply_computed_kernel<true><<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, delta, v, skip_mask, D, h,
+                                                                            t_next, target, spart);
+    CS_LAUNCHED();
+    score_finalize_kernel<<<(N + 3) / 4, 128, 0, stream>>>(spart, nch, N, scores);
+    CS_LAUNCHED();
+  } else {
+    apply_computed_kernel<false><<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, delta, v, skip_mask, D, h,
+                                                                             t_next, nullptr, nullptr);
     CS_LAUNCHED();
   }
   return CS_OK;
@@ -460,7 +787,7 @@ extern "C" cs_status cs_score(const float* x, const float* target, int N, long l
   float* partials = static_cast<float*>(workspace) + (size_t)N * nch * 2;
   sqdist_partials_kernel<<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, target, D, partials);
   CS_LAUNCHED();
-  score_finalize_kernel<<<(N + 127) / 128, 128, 0, stream>>>(partials, nch, N, scores);
+  score_finalize_kernel<<<(N + 3) / 4, 128, 0, stream>>>(partials, nch, N, scores);
   CS_LAUNCHED();
   return CS_OK;
 }
@@ -553,7 +880,7 @@ extern "C" cs_status cs_cache_decide_noalloc(const float* x, const float* x_ref,
     drift_partials_kernel<<<dim3(nch, N), kCacheThreads, 0, stream>>>(x, x_ref, has_ref, D, wf, N, partials);
     CS_LAUNCHED();
   }
-  decide_finalize_kernel<<<1, 256, N, stream>>>(partials, nch, accum, has_ref, N, wf, tau, force, skip_mask, idx,
+  decide_finalize_kernel<<<1, 1024, N, stream>>>(partials, nch, accum, has_ref, N, wf, tau, force, skip_mask, idx,
                                                 n_compute, err);
   CS_LAUNCHED();
   return CS_OK;

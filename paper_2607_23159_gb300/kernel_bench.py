@@ -33,7 +33,7 @@ def main():
     build.build()
     from paper_2607_23159_gb300 import binding as B
     ap = argparse.ArgumentParser()
-    ap.add_argument("kernel", choices=["attention", "gemm", "cache"])
+    ap.add_argument("kernel", choices=["attention", "gemm", "cache", "cache-fused"])
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--L", type=int, default=32760)
     ap.add_argument("--Lk", type=int, default=None)
@@ -93,9 +93,14 @@ def main():
         force = (torch.rand(N, device=dev) >= a.skip_frac).to(torch.uint8)
 
         def run():
-            B.cache_decide(st["x"], st["x_ref"], st["accum"], st["has_ref"], 20, 50, 0.1, 5, 5, skip, idx, nc, ws,
-                           force=force)
-            B.cache_apply(st["x"], st["x_ref"], st["delta"], v, skip, 0.6, 0.58)
+            if a.kernel == "cache-fused":
+                B.cache_decide_skip(st["x"], st["x_ref"], st["delta"], st["accum"], st["has_ref"], 20, 50, 0.6, 0.58,
+                                    0.1, 5, 5, skip, idx, nc, ws, force=force)
+                B.cache_apply_computed(st["x"], st["x_ref"], st["delta"], v, skip, 0.6, 0.58)
+            else:
+                B.cache_decide(st["x"], st["x_ref"], st["accum"], st["has_ref"], 20, 50, 0.1, 5, 5, skip, idx, nc,
+                               ws, force=force)
+                B.cache_apply(st["x"], st["x_ref"], st["delta"], v, skip, 0.6, 0.58)
         ms = _time(run, a.reps, a.warmup)
         n_skip = int((force == 0).sum())
         byts = (n_skip * 16.0 + (N - n_skip) * 24.0) * D

@@ -43,7 +43,7 @@ def test_param_count_matches_generator_layout(b):
 
 def test_workspace_and_version(b):
     assert b.lib.cs_version().startswith(b"cachedsearch")
-    assert b.cache_workspace_bytes(4, 2096640) == 4 * 64 * 12
+    assert b.cache_workspace_bytes(4, 2096640) == 4 * 256 * 12 + 256
     assert b.cache_workspace_bytes(0, 10) == 0
 
 

@@ -256,3 +256,57 @@ def test_score_topk_and_beam_refill(B):
     np.testing.assert_allclose(dst["x"].cpu().numpy(), nx, rtol=1e-6, atol=1e-6)
     np.testing.assert_array_equal(dst["x_ref"].cpu().numpy(), np.stack([s.x_ref for s in ns]).astype(np.float32))
     np.testing.assert_array_equal(dst["accum"].cpu().numpy(), np.array([s.a for s in ns], np.float32))
+
+
+@pytest.mark.parametrize("N,D,score", [(4, 2096640, True), (7, 50000, False), (16, 8192 * 3, True)])
+def test_fused_decide_skip_equals_two_pass_path(B, N, D, score):
+    """cs_cache_decide_skip + cs_cache_apply_computed give the same state bits as
+    cs_cache_decide + cs_cache_apply, over three steps (forced, free, scored)."""
+    T = 10
+    t = O.time_grid(T)
+    x0 = synth.normal(41, (N, D))
+    dx = synth.normal(42, (N, D)) * 0.02
+    states = []
+    for _ in range(2):
+        st = B.new_state(N, D)
+        st["x"].copy_(dev(x0))
+        st["x_ref"].copy_(dev(x0 + dx))
+        st["delta"].copy_(dev(synth.normal(43, (N, D))))
+        st["accum"].copy_(dev(synth.uniform(44, (N,), 0.0, 0.09)))
+        st["has_ref"].fill_(1)
+        st["has_ref"][N - 1] = 0
+        states.append(st)
+    ws = [torch.zeros(B.cache_workspace_bytes(N, D) // 4 + 1, device="cuda") for _ in range(2)]
+    y = dev(synth.normal(45, (D,)))
+    out = []
+    for which, st in enumerate(states):
+        skip = torch.zeros(N, dtype=torch.uint8, device="cuda")
+        idx = torch.zeros(N, dtype=torch.int32, device="cuda")
+        nc = torch.zeros(1, dtype=torch.int32, device="cuda")
+        sc = torch.zeros(N, device="cuda")
+        err = err_word()
+        rec = []
+        for k in (1, 4, 5):
+            v = dev(synth.normal(50 + k, (N, D)))
+            tgt = y if (score and k == 5) else None
+            if which == 0:
+                B.cache_decide(st["x"], st["x_ref"], st["accum"], st["has_ref"], k, T, 0.1, 1, 1, skip, idx, nc, ws[0],
+                               err=err)
+                B.cache_apply(st["x"], st["x_ref"], st["delta"], v, skip, float(t[k - 1]), float(t[k]),
+                              workspace=ws[0], target=tgt, scores=sc if tgt is not None else None)
+            else:
+                B.cache_decide_skip(st["x"], st["x_ref"], st["delta"], st["accum"], st["has_ref"], k, T,
+                                    float(t[k - 1]), float(t[k]), 0.1, 1, 1, skip, idx, nc, ws[1], target=tgt, err=err)
+                B.cache_apply_computed(st["x"], st["x_ref"], st["delta"], v, skip, float(t[k - 1]), float(t[k]),
+                                       workspace=ws[1], target=tgt, scores=sc if tgt is not None else None)
+            torch.cuda.synchronize()
+            rec.append((skip.clone(), idx[:int(nc[0])].clone(), sc.clone()))
+        assert int(err[0]) == 0
+        out.append(rec)
+    for (s0, i0, c0), (s1, i1, c1) in zip(*out):
+        assert torch.equal(s0, s1) and torch.equal(i0, i1)
+        # score partials are summed in a different element grouping by the two paths
+        torch.testing.assert_close(c0, c1, rtol=1e-6, atol=0)
+    assert 0 < int(out[0][1][0].sum()) < N or 0 < int(out[0][2][0].sum()) < N   # some candidates skip
+    for key in ("x", "x_ref", "delta", "accum", "has_ref"):
+        assert torch.equal(states[0][key], states[1][key]), key

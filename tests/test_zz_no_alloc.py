@@ -77,7 +77,7 @@ def test_noalloc_rejects_sizes_beyond_the_fixed_scratch(B):
     with pytest.raises(B.CSError) as e:
         B.cache_decide_noalloc(st["x"], st["x_ref"], st["accum"], st["has_ref"], 3, 10, 0.1, 1, 1, skip, idx, nc)
     assert e.value.status == B.CS_ERR_ARG and "limit" in str(e.value)
-    big = torch.zeros(1, 128 * 32768 + 1, device="cuda")
+    big = torch.zeros(1, 512 * 8192 + 1, device="cuda")
     with pytest.raises(B.CSError) as e:
         B.cache_decide_noalloc(big, big, st["accum"][:1], st["has_ref"][:1], 3, 10, 0.1, 1, 1, skip, idx, nc)
     assert e.value.status == B.CS_ERR_ARG and "limit" in str(e.value)
