@@ -48,7 +48,7 @@ struct AttnCfg {
   static constexpr int V_BYTES = 2 * VCH_BYTES;
   static constexpr int SLOT = K_BYTES > V_BYTES ? K_BYTES : V_BYTES;
   static constexpr int NSLOT = 4;
-  static constexpr int XBUF_BYTES = 2 * 2 * 2 * 128 * 4;   // [parity][tile][half][row] floats
+  static constexpr int XBUF_BYTES = 2 * 2 * 2 * 128 * 8;   // [parity][tile][half][row] tagged words
   static constexpr int SMEM = 2 * Q_BYTES + NSLOT * SLOT + XBUF_BYTES + 1024 + 256;
   static constexpr int THREADS = 18 * 32;
   static constexpr int OCOLS = HD >= 64 ? HD / 2 : HD;   // O columns each half-thread owns
@@ -66,7 +66,7 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;                                   // [2][Q_BYTES]
   uint8_t* sKV = sQ + 2 * Cfg::Q_BYTES;                 // [NSLOT][SLOT]
-  float* xbuf = reinterpret_cast<float*>(sKV + NS * Cfg::SLOT);
+  uint64_t* xbuf = reinterpret_cast<uint64_t*>(sKV + NS * Cfg::SLOT);
   uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(xbuf) + Cfg::XBUF_BYTES);
   uint64_t* q_full = bars;
   uint64_t* kv_full = bars + 1;            // [NS]
@@ -75,8 +75,7 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
   uint64_t* p_full = s_full + 2;           // [2]
   uint64_t* o_done = p_full + 2;           // [2]
   uint64_t* teardown = o_done + 2;
-  uint64_t* xbar = teardown + 1;           // [2][4]: the two warps of one row quarter
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(xbar + 8);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(teardown + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -98,10 +97,10 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
       mbar_init(&o_done[g], 1);
     }
     mbar_init(teardown, 1);
-    for (int i = 0; i < 8; ++i) mbar_init(&xbar[i], 64);
     *abort_flag = 0;
     fence_mbar_init();
   }
+  for (int i = threadIdx.x; i < Cfg::XBUF_BYTES / 8; i += blockDim.x) xbuf[i] = 0;   // tag 0: nothing yet
   if (warp == 1) {
     tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
@@ -149,23 +148,28 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       const uint32_t q_base = smem_u32(sQ);
+      // Descriptors are built once per tile; the k-th slice adds its byte offset / 16 to the
+      // start-address field (shared addresses stay below 2^18, so the field cannot carry).
+      // This thread shares its SMSP with four softmax warps, so every instruction per MMA counts.
       auto issue_s = [&](int g, uint32_t kslot) {
-        const uint32_t d = tmem_base + g * 128, a = q_base + g * Cfg::Q_BYTES;
+        const uint32_t d = tmem_base + g * 128;
+        const uint64_t ad = sdesc_sw128(q_base + g * Cfg::Q_BYTES), bd = sdesc_sw128(kslot);
 #pragma unroll
         for (int kk = 0; kk < Cfg::HDS / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * Cfg::CH_BYTES + (kk & 3) * 32;
-          umma_bf16_ss(d, sdesc_sw128(a + off), sdesc_sw128(kslot + off), Cfg::IDESC_S, kk > 0 ? 1u : 0u);
+          const uint64_t off = (uint64_t)(((kk >> 2) * Cfg::CH_BYTES + (kk & 3) * 32) >> 4);
+          umma_bf16_ss(d, ad + off, bd + off, Cfg::IDESC_S, kk > 0 ? 1u : 0u);
         }
         umma_commit(&s_full[g]);
       };
       auto issue_pv = [&](int g, uint32_t vslot, int j) {
         const uint32_t d = tmem_base + 256 + g * HD;
+        const uint32_t a0 = tmem_base + g * 128;
+        const uint64_t bd = sdesc_sw128(vslot);
 #pragma unroll
         for (int kk = 0; kk < Cfg::BKV / 16; ++kk) {
           // keys 16kk..16kk+15: half kk/4, packed bf16 pairs at columns 8*(kk%4) of that half
-          const uint32_t a = tmem_base + g * 128 + (kk >> 2) * 64 + (kk & 3) * 8;
-          const uint32_t offb = (kk >> 2) * Cfg::VCH_BYTES + (kk & 3) * 32;
-          umma_bf16_ts(d, a, sdesc_sw128(vslot + offb), Cfg::IDESC_O, (j > 0 || kk > 0) ? 1u : 0u);
+          const uint64_t offb = (uint64_t)(((kk >> 2) * Cfg::VCH_BYTES + (kk & 3) * 32) >> 4);
+          umma_bf16_ts(d, a0 + (kk >> 2) * 64 + (kk & 3) * 8, bd + offb, Cfg::IDESC_O, (j > 0 || kk > 0) ? 1u : 0u);
         }
         umma_commit(&o_done[g]);
       };
@@ -210,7 +214,6 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
     const int h = (sw >> 2) & 1;            // which 64 keys of each tile this thread takes
     const int qtr = warp & 3;               // TMEM lane quarter this warp may access
     const int r = qtr * 32 + lane;          // query row inside the tile
-    uint64_t* pair_bar = &xbar[g * 4 + qtr];   // the two warps of one row quarter
     const uint32_t lane_off = (uint32_t)(qtr * 32) << 16;
     const uint32_t tS = tmem_base + lane_off + g * 128 + h * 64;
     const uint32_t tO = tmem_base + lane_off + 256 + g * HD + h * Cfg::OCOLS;
@@ -238,11 +241,16 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
 #pragma unroll
         for (int q = 0; q < 4; ++q) mx[q] = fmax3(mx[q], __uint_as_float(u[e + 2 * q]), __uint_as_float(u[e + 2 * q + 1]));
       }
-      float* xb = xbuf + ((j & 1) * 2 + g) * 256;
-      xb[h * 128 + r] = fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
-      mbar_arrive(pair_bar);   // release: the partner sees this row max after its wait
-      if (!__all_sync(0xffffffffu, mbar_wait(pair_bar, j & 1, abort_flag, p.err))) { ok = false; break; }
-      const float rmax = fmaxf(xb[r], xb[128 + r]);
+      // row max of both halves: publish ours, read the partner's (tag j + 1)
+      uint64_t* xb = xbuf + ((j & 1) * 2 + g) * 256;
+      const float lmax = fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
+      xchg_put(xb + h * 128 + r, lmax, (uint32_t)j + 1);
+      float omax = 0.f;
+      if (!__all_sync(0xffffffffu, xchg_get(xb + (1 - h) * 128 + r, (uint32_t)j + 1, &omax, abort_flag, p.err))) {
+        ok = false;
+        break;
+      }
+      const float rmax = fmaxf(lmax, omax);
       const float m_new = fmaxf(m_run, rmax * sl2);
       const bool need = (j == 0) || (m_new > m_run + 8.f);
       const bool warp_need = __any_sync(0xffffffffu, need);
@@ -267,13 +275,9 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
       f2_unpack(acc[3], s6, s7);
       l_run = l_run * factor + (((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7)));
       m_run = m_use;
+      // PV of the previous tile has finished: the commit that signalled S(j) also covers
+      // every MMA issued before it, so O may be rescaled and P overwritten now
       if (j > 0) {
-        // PV of the previous tile must be done before O is rescaled and P overwritten
-        if (!__all_sync(0xffffffffu, mbar_wait(&o_done[g], (j - 1) & 1, abort_flag, p.err))) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
         if (warp_need && owns_o) {
 #pragma unroll 1
           for (int c = 0; c < Cfg::OCOLS / 32; ++c) {
@@ -293,13 +297,13 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
       mbar_arrive(&p_full[g]);
     }
     // final: row sum of both halves, then O / l -> bf16
-    float* xb = xbuf + ((nt & 1) * 2 + g) * 256;
-    xb[h * 128 + r] = l_run;
+    uint64_t* xb = xbuf + ((nt & 1) * 2 + g) * 256;
+    float l_oth = 0.f;
     if (ok) {
-      mbar_arrive(pair_bar);
-      ok = __all_sync(0xffffffffu, mbar_wait(pair_bar, nt & 1, abort_flag, p.err));
+      xchg_put(xb + h * 128 + r, l_run, (uint32_t)nt + 1);
+      ok = __all_sync(0xffffffffu, xchg_get(xb + (1 - h) * 128 + r, (uint32_t)nt + 1, &l_oth, abort_flag, p.err));
     }
-    const float l_tot = xb[r] + xb[128 + r];
+    const float l_tot = h == 0 ? l_run + l_oth : l_oth + l_run;
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&o_done[g], (nt - 1) & 1, abort_flag, p.err));
     if (ok && owns_o) {
       tc_fence_after();
