@@ -30,6 +30,7 @@ struct GemmArgs {
   __nv_bfloat16* k;
   __nv_bfloat16* vt;
   int L, d, heads, hd, hd_s, Lv, which_base;
+  int tma_out;   // float32 epilogues: stage in shared memory and TMA-store / TMA-reduce-add the output
   int* err;
 };
 
@@ -41,14 +42,23 @@ struct GemmCfg {
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int TMEM_COLS = 2 * BN;
-  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+  static constexpr int OUT_BYTES = 4 * 2 * 32 * 128;   // per epilogue warp: two 32 x 32 float32 staging buffers
+  static constexpr int SMEM = STAGES * STAGE_BYTES + OUT_BYTES + 1024 + 256;
   static constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
 };
+
+// tanh on the SFU (tanh.approx.f32: the hardware instruction, relative error ~2^-11, below
+// the bf16 rounding of the GELU output)
+__device__ __forceinline__ float tanh_approx(float x) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 
 __device__ __forceinline__ float gelu_tanh(float x) {
   // 0.5 x (1 + tanh(sqrt(2/pi) (x + 0.044715 x^3)))  (Hendrycks & Gimpel 2016)
   const float k0 = 0.7978845608028654f, k1 = 0.044715f;
-  return 0.5f * x * (1.f + tanhf(k0 * (x + k1 * x * x * x)));
+  return 0.5f * x * (1.f + tanh_approx(k0 * (x + k1 * x * x * x)));
 }
 
 // One thread's 32 consecutive accumulator columns [n, n+32) of row m.
@@ -144,14 +154,15 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& p, int m, int n, 
 template <int BN, int EPI>
 __global__ void __launch_bounds__(192, 1)
     gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                        const GemmArgs p) {
+                        const __grid_constant__ CUtensorMap tmC, const GemmArgs p) {
   using Cfg = GemmCfg<BN>;
   constexpr int BM = Cfg::BM, BK = Cfg::BK, STAGES = Cfg::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + STAGES * Cfg::A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * Cfg::STAGE_BYTES);
+  uint8_t* sOut = smem + STAGES * Cfg::STAGE_BYTES;   // 1024-aligned staging for float32 outputs
+  uint64_t* full = reinterpret_cast<uint64_t*>(sOut + Cfg::OUT_BYTES);
   uint64_t* empty = full + STAGES;
   uint64_t* tfull = empty + STAGES;
   uint64_t* tempty = tfull + 2;
@@ -252,18 +263,108 @@ __global__ void __launch_bounds__(192, 1)
     const int row = sp * 32 + lane;
     int acc = 0;
     uint32_t acc_phase = 0;
+    int nout = 0;   // chunks this warp has handed to TMA
+    if (lane == 0 && p.tma_out) tma_prefetch_desc(&tmC);
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
       if (!__all_sync(0xffffffffu, mbar_wait(&tfull[acc], acc_phase, abort_flag, p.err))) break;
       tc_fence_after();
       const int m0 = (tile / n_tiles) * BM, n0 = (tile % n_tiles) * BN;
       const int m = m0 + row;
       const uint32_t tbase = tmem_base + ((uint32_t)(sp * 32) << 16) + acc * BN;
+      if constexpr (EPI == CS_EPI_BF16 || EPI == CS_EPI_GELU_BF16) {
+        if (p.tma_out) {
+          // 64 columns at a time: 32 rows x 128 B of bf16 per warp -> staging -> one TMA store
+#pragma unroll 1
+          for (int c = 0; c < BN / 64; ++c) {
+            const int n = n0 + c * 64;
+            if (n >= p.N) break;   // uniform across the warp
+            uint32_t r0[32], r1[32];
+            tmem_ld32(tbase + c * 64, r0);
+            tmem_ld32(tbase + c * 64 + 32, r1);
+            uint8_t* buf = sOut + (sp * 2 + (nout & 1)) * 4096;
+            if (lane == 0 && nout >= 2) bulk_wait_read_1();
+            __syncwarp();
+            const float4* b4 = p.bias ? reinterpret_cast<const float4*>(p.bias + n) : nullptr;
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+              float v[8];
+#pragma unroll
+              for (int j = 0; j < 8; ++j) v[j] = __uint_as_float(u < 4 ? r0[8 * u + j] : r1[8 * (u - 4) + j]);
+              if (b4) {
+                const float4 ba = __ldg(b4 + 2 * u), bb = __ldg(b4 + 2 * u + 1);
+                v[0] += ba.x; v[1] += ba.y; v[2] += ba.z; v[3] += ba.w;
+                v[4] += bb.x; v[5] += bb.y; v[6] += bb.z; v[7] += bb.w;
+              }
+              if constexpr (EPI == CS_EPI_GELU_BF16) {
+#pragma unroll
+                for (int j = 0; j < 8; ++j) v[j] = gelu_tanh(v[j]);
+              }
+              uint4 w;
+              w.x = pack_bf16x2(v[0], v[1]);
+              w.y = pack_bf16x2(v[2], v[3]);
+              w.z = pack_bf16x2(v[4], v[5]);
+              w.w = pack_bf16x2(v[6], v[7]);
+              *reinterpret_cast<uint4*>(buf + lane * 128 + ((u ^ (lane & 7)) << 4)) = w;
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(&tmC, buf, n, m0 + sp * 32);
+              bulk_commit();
+            }
+            ++nout;
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&tempty[acc]);
+          acc ^= 1;
+          if (acc == 0) acc_phase ^= 1;
+          continue;
+        }
+      }
 #pragma unroll 1
       for (int c = 0; c < BN / 32; ++c) {
         const int n = n0 + c * 32;
         if (n >= p.N) break;   // uniform across the warp
         uint32_t r[32];
         tmem_ld32(tbase + c * 32, r);
+        if constexpr (EPI == CS_EPI_F32 || EPI == CS_EPI_RESID_F32) {
+          if (p.tma_out) {
+            // this warp's 32 rows x 32 columns -> 128-byte-swizzled staging -> one TMA op
+            // (a plain store, or for the residual an add performed in L2)
+            uint8_t* buf = sOut + (sp * 2 + (nout & 1)) * 4096;
+            if (lane == 0 && nout >= 2) bulk_wait_read_1();   // the op that last read this buffer is done
+            __syncwarp();
+            float f[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) f[j] = __uint_as_float(r[j]);
+            const float4* b4 = p.bias ? reinterpret_cast<const float4*>(p.bias + n) : nullptr;
+            const float4* g4 = (EPI == CS_EPI_RESID_F32 && p.gate) ? reinterpret_cast<const float4*>(p.gate + n)
+                                                                   : nullptr;
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+              float4 v = make_float4(f[4 * u], f[4 * u + 1], f[4 * u + 2], f[4 * u + 3]);
+              if (b4) {
+                const float4 b = __ldg(b4 + u);
+                v.x += b.x; v.y += b.y; v.z += b.z; v.w += b.w;
+              }
+              if (g4) {
+                const float4 g = __ldg(g4 + u);
+                v.x *= g.x; v.y *= g.y; v.z *= g.z; v.w *= g.w;
+              }
+              *reinterpret_cast<float4*>(buf + lane * 128 + ((u ^ (lane & 7)) << 4)) = v;
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              if constexpr (EPI == CS_EPI_RESID_F32) tma_reduce_add_2d(&tmC, buf, n, m0 + sp * 32);
+              else tma_store_2d(&tmC, buf, n, m0 + sp * 32);
+              bulk_commit();
+            }
+            ++nout;
+            continue;
+          }
+        }
         if (m < p.M) epilogue_chunk<EPI>(p, m, n, r);
       }
       tc_fence_before();
@@ -272,6 +373,7 @@ __global__ void __launch_bounds__(192, 1)
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1;
     }
+    if (lane == 0 && nout > 0) bulk_wait_all();   // output writes complete before the CTA exits
   }
 
   tc_fence_before();
@@ -293,11 +395,31 @@ static cs_status launch_gemm(const void* A, const void* B, const GemmArgs& args,
   const uint64_t db[2] = {(uint64_t)args.K, (uint64_t)args.N};
   const uint32_t bb[2] = {64, (uint32_t)BN};
   CS_TRY(make_tmap_bf16(&tb, B, 2, db, sa, bb));
+  // float32 outputs go through TMA when the output rows are TMA-addressable
+  GemmArgs a = args;
+  CUtensorMap tc = ta;   // unused unless a.tma_out
+  a.tma_out = 0;
+  if ((EPI == CS_EPI_F32 || EPI == CS_EPI_RESID_F32) && (args.N % 32) == 0 && (args.ldo % 4) == 0 &&
+      (reinterpret_cast<uintptr_t>(args.out) & 15) == 0) {
+    const uint64_t dc[2] = {(uint64_t)args.N, (uint64_t)args.M};
+    const uint64_t sc[1] = {(uint64_t)args.ldo * 4};
+    const uint32_t bc[2] = {32, 32};
+    CS_TRY(make_tmap(&tc, args.out, 2, dc, sc, bc, true));
+    a.tma_out = 1;
+  }
+  if ((EPI == CS_EPI_BF16 || EPI == CS_EPI_GELU_BF16) && (args.N % 64) == 0 && (args.ldo % 8) == 0 &&
+      (reinterpret_cast<uintptr_t>(args.out) & 15) == 0) {
+    const uint64_t dc[2] = {(uint64_t)args.N, (uint64_t)args.M};
+    const uint64_t sc[1] = {(uint64_t)args.ldo * 2};
+    const uint32_t bc[2] = {64, 32};
+    CS_TRY(make_tmap(&tc, args.out, 2, dc, sc, bc, false));
+    a.tma_out = 1;
+  }
   auto kern = gemm_tcgen05_kernel<BN, EPI>;
   CS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
   const int tiles = ((args.M + 127) / 128) * ((args.N + BN - 1) / BN);
   const int grid = tiles < num_sms() ? tiles : num_sms();
-  kern<<<grid, 192, Cfg::SMEM, stream>>>(ta, tb, args);
+  kern<<<grid, 192, Cfg::SMEM, stream>>>(ta, tb, tc, a);
   CS_LAUNCHED();
   return CS_OK;
 }
