@@ -33,7 +33,7 @@ def main():
     build.build()
     from paper_2607_23159_gb300 import binding as B
     ap = argparse.ArgumentParser()
-    ap.add_argument("kernel", choices=["attention", "gemm", "cache", "cache-fused"])
+    ap.add_argument("kernel", choices=["attention", "gemm", "qkv", "layernorm", "cache", "cache-fused"])
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--L", type=int, default=32760)
     ap.add_argument("--Lk", type=int, default=None)
@@ -78,6 +78,25 @@ def main():
         ms = _time(lambda: B.gemm(A, W, a.epi, C, bias=bias), a.reps, a.warmup)
         out.update(shape=dict(M=a.M, N=a.N, K=a.K, epi=a.epi), ms=ms,
                    tflops=2.0 * a.M * a.N * a.K / (ms / 1e3) / 1e12)
+    elif a.kernel == "qkv":
+        # QKV projection with the per-head Q/K and transposed V scatter; M = batch * L rows
+        M, d = a.batch * a.L, a.heads * a.hd
+        A = torch.randn(M, a.K, device=dev).to(bf)
+        W = (torch.randn(3 * d, a.K, device=dev) * 0.05).to(bf)
+        bias = torch.zeros(3 * d, device=dev)
+        hds, Lv = max(a.hd, 64), (a.L + 7) // 8 * 8
+        q = torch.zeros(a.batch * a.heads, a.L, hds, device=dev, dtype=bf)
+        k = torch.zeros_like(q)
+        vt = torch.zeros(a.batch * a.heads, a.hd, Lv, device=dev, dtype=bf)
+        ms = _time(lambda: B.gemm_qkv(A, W, bias, a.L, d, a.heads, 0, q, k, vt, Lv), a.reps, a.warmup)
+        out.update(shape=dict(M=M, N=3 * d, K=a.K), ms=ms, tflops=2.0 * M * 3 * d * a.K / (ms / 1e3) / 1e12)
+    elif a.kernel == "layernorm":
+        M, d = a.M, a.K
+        x = torch.randn(M, d, device=dev)
+        sh, sc = torch.randn(d, device=dev), torch.randn(d, device=dev)
+        o = torch.empty(M, d, device=dev, dtype=bf)
+        ms = _time(lambda: B.layernorm_modulate(x, sh, sc, o), a.reps, a.warmup)
+        out.update(shape=dict(M=M, d=d), ms=ms, gbs=M * d * 6.0 / (ms / 1e3) / 1e9)
     else:
         N, D = a.N, a.D
         st = B.new_state(N, D)
