@@ -2,20 +2,24 @@
 // the DiT blocks).  One CTA takes 256 query rows of one (batch item, head) as two
 // 128-row tiles A and B and streams the keys in tiles of 128:
 //
-//   warp 0       TMA producer: Q once, then K_j and V_j^T tiles through a 4-slot ring
+//   warp 0       TMA producer: Q once, then stages {V_{j-1}^T, K_j} through a 2-stage ring
 //   warp 1       TMEM allocator + MMA issuer, in the order
 //                  S_A(0) S_B(0) | PV_A(j) S_A(j+1) PV_B(j) S_B(j+1) | ...
 //                so that the tensor core works on one tile while the other's softmax runs
-//   warps 2..9   softmax of tile A, warps 10..17 softmax of tile B.  Two threads share a
-//                query row (warps w and w+4 read the same TMEM lanes): each takes 64 of the
-//                128 keys, the two exchange their row maxima through shared memory and a
-//                named barrier, and keep separate partial row sums until the end.  Online
-//                softmax in log2 units with lazy O rescaling (only when the running max
-//                grows by more than 8).  P is written back to TMEM as bf16 over the
-//                thread's own S columns and fed to the PV MMA as the TMEM A operand.
+//   warps 2..5   softmax of tile A, warps 6..9 softmax of tile B: one thread per query
+//                row (the warp's TMEM lane quarter), all 128 keys of the tile in
+//                registers.  Online softmax in log2 units with lazy O rescaling (only
+//                when the running max grows by more than 8).  P is written back to TMEM
+//                as bf16 over the row's own S columns and fed to the PV MMA as the TMEM
+//                A operand.
 //
-// TMEM (512 columns): S_A [0,128), S_B [128,256) (P_g aliases the first 32 columns of
-// each 64-key half of S_g), O_A [256, 256+hd), O_B [256+hd, 256+2hd).  V is stored
+// One softmax warp per tile on each SM sub-partition: a tcgen05.mma needs issue slots on
+// the issuer's sub-partition, and measured on GB300 the tensor core keeps its rate next
+// to one busy warp but drops to ~70 % of it next to two or more (the layout with two
+// threads per row, 18 warps, ran its N=128 MMAs at ~90 cycles instead of 64).
+//
+// TMEM (512 columns): S_A [0,128), S_B [128,256) (P_g, keys 64h..64h+63 packed in pairs,
+// aliases columns [64h, 64h+32) of S_g), O_A [256, 256+hd), O_B [256+hd, 256+2hd).  V is stored
 // transposed (V^T [hd][keys]) so that it is a K-major B operand in shared memory.
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -47,11 +51,9 @@ struct AttnCfg {
   static constexpr int VCH_BYTES = HD * 64 * 2;    // one [hd x 64 keys] chunk of V^T
   static constexpr int V_BYTES = 2 * VCH_BYTES;
   static constexpr int SLOT = K_BYTES > V_BYTES ? K_BYTES : V_BYTES;
-  static constexpr int NSLOT = 4;
-  static constexpr int XBUF_BYTES = 2 * 2 * 2 * 128 * 8;   // [parity][tile][half][row] tagged words
-  static constexpr int SMEM = 2 * Q_BYTES + NSLOT * SLOT + XBUF_BYTES + 1024 + 256;
-  static constexpr int THREADS = 18 * 32;
-  static constexpr int OCOLS = HD >= 64 ? HD / 2 : HD;   // O columns each half-thread owns
+  static constexpr int NSTAGE = 2;                  // ring stages, each a V slot and a K slot
+  static constexpr int SMEM = 2 * Q_BYTES + NSTAGE * 2 * SLOT + 1024 + 256;
+  static constexpr int THREADS = 10 * 32;
   static constexpr uint32_t IDESC_S = idesc_bf16_f32(128, BKV);
   static constexpr uint32_t IDESC_O = idesc_bf16_f32(128, HD);
 };
@@ -61,13 +63,12 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
     attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                         const __grid_constant__ CUtensorMap tmV, const AttnArgs p) {
   using Cfg = AttnCfg<HD>;
-  constexpr int NS = Cfg::NSLOT;
+  constexpr int NS = Cfg::NSTAGE;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;                                   // [2][Q_BYTES]
-  uint8_t* sKV = sQ + 2 * Cfg::Q_BYTES;                 // [NSLOT][SLOT]
-  uint64_t* xbuf = reinterpret_cast<uint64_t*>(sKV + NS * Cfg::SLOT);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(xbuf) + Cfg::XBUF_BYTES);
+  uint8_t* sKV = sQ + 2 * Cfg::Q_BYTES;                 // [NSTAGE][V slot, K slot][SLOT]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + NS * 2 * Cfg::SLOT);
   uint64_t* q_full = bars;
   uint64_t* kv_full = bars + 1;            // [NS]
   uint64_t* kv_empty = kv_full + NS;       // [NS]
@@ -93,14 +94,13 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
     }
     for (int g = 0; g < 2; ++g) {
       mbar_init(&s_full[g], 1);
-      mbar_init(&p_full[g], 256);
+      mbar_init(&p_full[g], 128);
       mbar_init(&o_done[g], 1);
     }
     mbar_init(teardown, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
-  for (int i = threadIdx.x; i < Cfg::XBUF_BYTES / 8; i += blockDim.x) xbuf[i] = 0;   // tag 0: nothing yet
   if (warp == 1) {
     tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
@@ -120,28 +120,27 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
       for (int g = 0; g < 2; ++g)
         for (int c = 0; c < Cfg::QCH; ++c)
           tma_load_3d(sQ + g * Cfg::Q_BYTES + c * Cfg::CH_BYTES, &tmQ, q_full, c * 64, q0 + g * 128, bh);
+      // stage st holds V_{st-1} (st >= 1) and K_st (st < nt): exactly what the MMAs issued
+      // after P(st-1) read, so the issuer waits on one barrier per key tile
       int issued = 0;
-      for (int s = 0; s < 2 * nt; ++s) {
-        const int slot = s % NS;
-        const uint32_t ph = (s / NS) & 1;
-        if (!mbar_wait(&kv_empty[slot], ph ^ 1, abort_flag, p.err)) break;
-        uint8_t* dst = sKV + slot * Cfg::SLOT;
-        const int j = s >> 1;
-        if ((s & 1) == 0) {
-          mbar_arrive_expect_tx(&kv_full[slot], Cfg::K_BYTES);
+      for (int st = 0; st <= nt; ++st) {
+        const int b = st % NS;
+        if (!mbar_wait(&kv_empty[b], ((st / NS) & 1) ^ 1, abort_flag, p.err)) break;
+        uint8_t* dv = sKV + b * 2 * Cfg::SLOT;
+        uint8_t* dk = dv + Cfg::SLOT;
+        mbar_arrive_expect_tx(&kv_full[b], (st >= 1 ? Cfg::V_BYTES : 0) + (st < nt ? Cfg::K_BYTES : 0));
+        if (st < nt)
           for (int c = 0; c < Cfg::QCH; ++c)
-            tma_load_3d(dst + c * Cfg::CH_BYTES, &tmK, &kv_full[slot], c * 64, j * Cfg::BKV, bkv);
-        } else {
-          mbar_arrive_expect_tx(&kv_full[slot], Cfg::V_BYTES);
+            tma_load_3d(dk + c * Cfg::CH_BYTES, &tmK, &kv_full[b], c * 64, st * Cfg::BKV, bkv);
+        if (st >= 1)
           for (int c = 0; c < 2; ++c)
-            tma_load_3d(dst + c * Cfg::VCH_BYTES, &tmV, &kv_full[slot], j * Cfg::BKV + c * 64, 0, bkv);
-        }
-        issued = s + 1;
+            tma_load_3d(dv + c * Cfg::VCH_BYTES, &tmV, &kv_full[b], (st - 1) * Cfg::BKV + c * 64, 0, bkv);
+        issued = st + 1;
       }
       if (*abort_flag) {
         mbar_wait_teardown(q_full, 0);
-        for (int s = issued - NS < 0 ? 0 : issued - NS; s < issued; ++s)
-          mbar_wait_teardown(&kv_full[s % NS], (s / NS) & 1);
+        for (int st = issued - NS < 0 ? 0 : issued - NS; st < issued; ++st)
+          mbar_wait_teardown(&kv_full[st % NS], (st / NS) & 1);
       }
     }
   } else if (warp == 1) {
@@ -150,7 +149,9 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
       const uint32_t q_base = smem_u32(sQ);
       // Descriptors are built once per tile; the k-th slice adds its byte offset / 16 to the
       // start-address field (shared addresses stay below 2^18, so the field cannot carry).
-      // This thread shares its SMSP with four softmax warps, so every instruction per MMA counts.
+      // A tcgen05.mma stream must not pause: each wait or fence between two MMAs costs the
+      // tensor core ~100-200 cycles (measured on GB300), so a key tile takes three waits:
+      // its K/V stage, P_A and P_B.
       auto issue_s = [&](int g, uint32_t kslot) {
         const uint32_t d = tmem_base + g * 128;
         const uint64_t ad = sdesc_sw128(q_base + g * Cfg::Q_BYTES), bd = sdesc_sw128(kslot);
@@ -171,36 +172,31 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
           const uint64_t offb = (uint64_t)(((kk >> 2) * Cfg::VCH_BYTES + (kk & 3) * 32) >> 4);
           umma_bf16_ts(d, a0 + (kk >> 2) * 64 + (kk & 3) * 8, bd + offb, Cfg::IDESC_O, (j > 0 || kk > 0) ? 1u : 0u);
         }
-        umma_commit(&o_done[g]);
+        umma_commit(&o_done[g]);   // measured: this commit after each PV group runs faster than none
       };
-      auto slot_addr = [&](int s) { return smem_u32(sKV + (s % NS) * Cfg::SLOT); };
+      auto v_addr = [&](int st) { return smem_u32(sKV + (st % NS) * 2 * Cfg::SLOT); };
+      auto k_addr = [&](int st) { return v_addr(st) + Cfg::SLOT; };
       bool ok = mbar_wait(q_full, 0, abort_flag, p.err);
       if (ok) ok = mbar_wait(&kv_full[0], 0, abort_flag, p.err);
       if (ok) {
         tc_fence_after();
-        issue_s(0, slot_addr(0));
-        issue_s(1, slot_addr(0));
+        issue_s(0, k_addr(0));
+        issue_s(1, k_addr(0));
         umma_commit(&kv_empty[0]);
       }
       for (int j = 0; ok && j < nt; ++j) {
-        const int sv = 2 * j + 1, sk = 2 * j + 2;
-        if (!mbar_wait(&kv_full[sv % NS], (sv / NS) & 1, abort_flag, p.err)) break;
+        const int st = j + 1;
+        const bool more = j + 1 < nt;
+        if (!mbar_wait(&kv_full[st % NS], (st / NS) & 1, abort_flag, p.err)) break;
         if (!mbar_wait(&p_full[0], j & 1, abort_flag, p.err)) break;
         tc_fence_after();
-        issue_pv(0, slot_addr(sv), j);
-        if (j + 1 < nt) {
-          if (!mbar_wait(&kv_full[sk % NS], (sk / NS) & 1, abort_flag, p.err)) break;
-          tc_fence_after();
-          issue_s(0, slot_addr(sk));
-        }
+        issue_pv(0, v_addr(st), j);
+        if (more) issue_s(0, k_addr(st));
         if (!mbar_wait(&p_full[1], j & 1, abort_flag, p.err)) break;
         tc_fence_after();
-        issue_pv(1, slot_addr(sv), j);
-        umma_commit(&kv_empty[sv % NS]);
-        if (j + 1 < nt) {
-          issue_s(1, slot_addr(sk));
-          umma_commit(&kv_empty[sk % NS]);
-        }
+        issue_pv(1, v_addr(st), j);
+        if (more) issue_s(1, k_addr(st));
+        umma_commit(&kv_empty[st % NS]);
       }
       if (*abort_flag) {
         umma_commit(teardown);
@@ -209,15 +205,12 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ softmax
-    const int sw = warp - 2;
-    const int g = sw >> 3;                  // query tile: 0 = A (warps 2..9), 1 = B (warps 10..17)
-    const int h = (sw >> 2) & 1;            // which 64 keys of each tile this thread takes
+    const int g = (warp - 2) >> 2;          // query tile: 0 = A (warps 2..5), 1 = B (warps 6..9)
     const int qtr = warp & 3;               // TMEM lane quarter this warp may access
     const int r = qtr * 32 + lane;          // query row inside the tile
     const uint32_t lane_off = (uint32_t)(qtr * 32) << 16;
-    const uint32_t tS = tmem_base + lane_off + g * 128 + h * 64;
-    const uint32_t tO = tmem_base + lane_off + 256 + g * HD + h * Cfg::OCOLS;
-    const bool owns_o = (HD >= 64) || (h == 0);
+    const uint32_t tS = tmem_base + lane_off + g * 128;
+    const uint32_t tO = tmem_base + lane_off + 256 + g * HD;
     const float sl2 = p.scale_log2;
     const uint64_t sc2 = f2_pack(sl2, sl2);
     float m_run = -INFINITY, l_run = 0.f;
@@ -225,94 +218,74 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
     for (int j = 0; j < nt; ++j) {
       if (!__all_sync(0xffffffffu, mbar_wait(&s_full[g], j & 1, abort_flag, p.err))) { ok = false; break; }
       tc_fence_after();
-      uint32_t u[64];
-      tmem_ld64(tS, u);
-      const int valid = p.Lk - j * Cfg::BKV - h * 64;
-      if (valid < 64) {
+      uint32_t u[128];
+      tmem_ld128(tS, u);
+      const int valid = p.Lk - j * Cfg::BKV;
+      if (valid < Cfg::BKV) {
 #pragma unroll
-        for (int e = 0; e < 64; ++e)
+        for (int e = 0; e < Cfg::BKV; ++e)
           if (e >= valid) u[e] = __float_as_uint(-INFINITY);
       }
       float mx[4];
 #pragma unroll
       for (int q = 0; q < 4; ++q) mx[q] = __uint_as_float(u[q]);
 #pragma unroll
-      for (int e = 4; e < 64; e += 8) {
+      for (int e = 4; e < Cfg::BKV - 4; e += 8) {
 #pragma unroll
         for (int q = 0; q < 4; ++q) mx[q] = fmax3(mx[q], __uint_as_float(u[e + 2 * q]), __uint_as_float(u[e + 2 * q + 1]));
       }
-      // row max of both halves: publish ours, read the partner's (tag j + 1)
-      uint64_t* xb = xbuf + ((j & 1) * 2 + g) * 256;
-      const float lmax = fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
-      xchg_put(xb + h * 128 + r, lmax, (uint32_t)j + 1);
-      float omax = 0.f;
-      if (!__all_sync(0xffffffffu, xchg_get(xb + (1 - h) * 128 + r, (uint32_t)j + 1, &omax, abort_flag, p.err))) {
-        ok = false;
-        break;
-      }
-      const float rmax = fmaxf(lmax, omax);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) mx[q] = fmaxf(mx[q], __uint_as_float(u[Cfg::BKV - 4 + q]));
+      const float rmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
       const float m_new = fmaxf(m_run, rmax * sl2);
       const bool need = (j == 0) || (m_new > m_run + 8.f);
       const bool warp_need = __any_sync(0xffffffffu, need);
       const float m_use = need ? m_new : m_run;
       const float factor = need ? ex2_approx(m_run - m_use) : 1.f;
       const uint64_t nm2 = f2_pack(-m_use, -m_use);
-      // p = 2^(s * scale * log2(e) - m) on pairs; P packed as bf16 pairs in place
-      uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
+      // p = 2^(s * scale * log2(e) - m) on pairs; P packed as bf16 pairs in place (u[0..63])
+      uint64_t acc[2] = {0ull, 0ull};
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
+      for (int i = 0; i < Cfg::BKV / 2; ++i) {
         float a, b;
         f2_unpack(f2_fma(f2_pack(__uint_as_float(u[2 * i]), __uint_as_float(u[2 * i + 1])), sc2, nm2), a, b);
         a = ex2_approx(a);
         b = ex2_approx(b);
-        acc[i & 3] = f2_add(acc[i & 3], f2_pack(a, b));
+        acc[i & 1] = f2_add(acc[i & 1], f2_pack(a, b));
         u[i] = pack_bf16x2(a, b);
       }
-      float s0, s1, s2, s3, s4, s5, s6, s7;
+      float s0, s1, s2, s3;
       f2_unpack(acc[0], s0, s1);
       f2_unpack(acc[1], s2, s3);
-      f2_unpack(acc[2], s4, s5);
-      f2_unpack(acc[3], s6, s7);
-      l_run = l_run * factor + (((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7)));
+      l_run = l_run * factor + ((s0 + s1) + (s2 + s3));
       m_run = m_use;
       // PV of the previous tile has finished: the commit that signalled S(j) also covers
       // every MMA issued before it, so O may be rescaled and P overwritten now
-      if (j > 0) {
-        if (warp_need && owns_o) {
+      if (j > 0 && warp_need) {
 #pragma unroll 1
-          for (int c = 0; c < Cfg::OCOLS / 32; ++c) {
-            uint32_t o[32];
-            tmem_ld32(tO + c * 32, o);
+        for (int c = 0; c < HD / 32; ++c) {
+          uint32_t o[32];
+          tmem_ld32(tO + c * 32, o);
 #pragma unroll
-            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * factor);
-            tmem_st32(tO + c * 32, o);
-          }
+          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * factor);
+          tmem_st32(tO + c * 32, o);
         }
       }
-      uint32_t pk[32];
-#pragma unroll
-      for (int i = 0; i < 32; ++i) pk[i] = u[i];
-      tmem_st32(tS, pk);
+      tmem_st32(tS, *reinterpret_cast<const uint32_t(*)[32]>(&u[0]));
+      tmem_st32(tS + 64, *reinterpret_cast<const uint32_t(*)[32]>(&u[32]));
       tc_fence_before();
       mbar_arrive(&p_full[g]);
     }
-    // final: row sum of both halves, then O / l -> bf16
-    uint64_t* xb = xbuf + ((nt & 1) * 2 + g) * 256;
-    float l_oth = 0.f;
-    if (ok) {
-      xchg_put(xb + h * 128 + r, l_run, (uint32_t)nt + 1);
-      ok = __all_sync(0xffffffffu, xchg_get(xb + (1 - h) * 128 + r, (uint32_t)nt + 1, &l_oth, abort_flag, p.err));
-    }
-    const float l_tot = h == 0 ? l_run + l_oth : l_oth + l_run;
+    // final: O / l -> bf16
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&o_done[g], (nt - 1) & 1, abort_flag, p.err));
-    if (ok && owns_o) {
+    if (ok) {
       tc_fence_after();
       const int q = q0 + g * 128 + r;
-      const float inv_l = 1.f / l_tot;
+      const float inv_l = 1.f / l_run;
       const int d = p.heads * HD;
-      __nv_bfloat16* orow = p.o + ((long long)jb * p.Lq + q) * d + head * HD + h * Cfg::OCOLS;
+      __nv_bfloat16* orow = p.o + ((long long)jb * p.Lq + q) * d + head * HD;
 #pragma unroll 1
-      for (int c = 0; c < Cfg::OCOLS / 32; ++c) {
+      for (int c = 0; c < HD / 32; ++c) {
         uint32_t u[32];
         tmem_ld32(tO + c * 32, u);
         if (q < p.Lq) {
