@@ -3,8 +3,9 @@
 // 128-row tiles A and B and streams the keys in tiles of 128:
 //
 //   warp 0       TMA producer: Q once, then stages {V_{j-1}^T, K_j} through a 2-stage ring
-//   warp 1       TMEM allocator + MMA issuer, in the order
-//                  S_A(0) S_B(0) | PV_A(j) S_A(j+1) PV_B(j) S_B(j+1) | ...
+//   warp 1       TMEM allocator + MMA issuer of tile A, warp 10 MMA issuer of tile B;
+//                a token alternates them, giving the order
+//                  S_A(0) S_B(0) | PV_A(j) S_A(j+1) | PV_B(j) S_B(j+1) | ...
 //                so that the tensor core works on one tile while the other's softmax runs
 //   warps 2..5   softmax of tile A, warps 6..9 softmax of tile B: one thread per query
 //                row (the warp's TMEM lane quarter), all 128 keys of the tile in
@@ -53,7 +54,9 @@ struct AttnCfg {
   static constexpr int SLOT = K_BYTES > V_BYTES ? K_BYTES : V_BYTES;
   static constexpr int NSTAGE = 2;                  // ring stages, each a V slot and a K slot
   static constexpr int SMEM = 2 * Q_BYTES + NSTAGE * 2 * SLOT + 1024 + 256;
-  static constexpr int THREADS = 10 * 32;
+  static constexpr int ISSUER_B = 10;                 // second MMA issuer (another sub-partition)
+  static constexpr int HANDOVER = 4;                  // MMAs left in a group when the token passes (3-6 measured best)
+  static constexpr int THREADS = 11 * 32;
   static constexpr uint32_t IDESC_S = idesc_bf16_f32(128, BKV);
   static constexpr uint32_t IDESC_O = idesc_bf16_f32(128, HD);
 };
@@ -75,8 +78,9 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
   uint64_t* s_full = kv_empty + NS;        // [2]
   uint64_t* p_full = s_full + 2;           // [2]
   uint64_t* o_done = p_full + 2;           // [2]
-  uint64_t* teardown = o_done + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(teardown + 1);
+  uint64_t* tok = o_done + 2;              // [2]: tok[g] = tile g may start its next MMA group
+  uint64_t* teardown = tok + 2;            // [2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(teardown + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -90,14 +94,17 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
     mbar_init(q_full, 1);
     for (int s = 0; s < NS; ++s) {
       mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
+      mbar_init(&kv_empty[s], 2);          // both issuers read every stage
     }
     for (int g = 0; g < 2; ++g) {
       mbar_init(&s_full[g], 1);
       mbar_init(&p_full[g], 128);
       mbar_init(&o_done[g], 1);
     }
-    mbar_init(teardown, 1);
+    for (int g = 0; g < 2; ++g) {
+      mbar_init(&tok[g], 1);
+      mbar_init(&teardown[g], 1);
+    }
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -143,64 +150,76 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
           mbar_wait_teardown(&kv_full[st % NS], (st / NS) & 1);
       }
     }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (warp == 1 || warp == Cfg::ISSUER_B) {
+    // ------------------------------------------------------------ MMA issuers
+    // One issuing thread per query tile, on different SM sub-partitions, handing a token
+    // back and forth so that the tensor core sees the groups in the order
+    //   S_A(0) S_B(0) | PV_A(j) S_A(j+1) | PV_B(j) S_B(j+1) | ...
+    // A tcgen05.mma stream must not pause (measured on GB300: each wait or fence between
+    // two MMAs costs the tensor core ~100-200 cycles).  The token is handed over HANDOVER
+    // MMAs before the end of a group, so the next group's waits and fence run while those
+    // MMAs execute.  Each thread's MMAs run in its issue order, which is all that a tile's
+    // TMEM reuse needs (PV_g(j) reads P_g(j) before S_g(j+1) overwrites it).
     if (lane == 0) {
+      const int g = warp == 1 ? 0 : 1;
       const uint32_t q_base = smem_u32(sQ);
+      const uint32_t sdst = tmem_base + g * 128, odst = tmem_base + 256 + g * HD;
+      const uint64_t ad = sdesc_sw128(q_base + g * Cfg::Q_BYTES);
       // Descriptors are built once per tile; the k-th slice adds its byte offset / 16 to the
       // start-address field (shared addresses stay below 2^18, so the field cannot carry).
-      // A tcgen05.mma stream must not pause: each wait or fence between two MMAs costs the
-      // tensor core ~100-200 cycles (measured on GB300), so a key tile takes three waits:
-      // its K/V stage, P_A and P_B.
-      auto issue_s = [&](int g, uint32_t kslot) {
-        const uint32_t d = tmem_base + g * 128;
-        const uint64_t ad = sdesc_sw128(q_base + g * Cfg::Q_BYTES), bd = sdesc_sw128(kslot);
+      auto issue_s = [&](uint32_t kslot, uint64_t* pass) {
+        const uint64_t bd = sdesc_sw128(kslot);
 #pragma unroll
         for (int kk = 0; kk < Cfg::HDS / 16; ++kk) {
+          if (pass && kk == Cfg::HDS / 16 - Cfg::HANDOVER) mbar_arrive(pass);
           const uint64_t off = (uint64_t)(((kk >> 2) * Cfg::CH_BYTES + (kk & 3) * 32) >> 4);
-          umma_bf16_ss(d, ad + off, bd + off, Cfg::IDESC_S, kk > 0 ? 1u : 0u);
+          umma_bf16_ss(sdst, ad + off, bd + off, Cfg::IDESC_S, kk > 0 ? 1u : 0u);
         }
         umma_commit(&s_full[g]);
       };
-      auto issue_pv = [&](int g, uint32_t vslot, int j) {
-        const uint32_t d = tmem_base + 256 + g * HD;
-        const uint32_t a0 = tmem_base + g * 128;
+      auto issue_pv = [&](uint32_t vslot, int j, uint64_t* pass) {
         const uint64_t bd = sdesc_sw128(vslot);
 #pragma unroll
         for (int kk = 0; kk < Cfg::BKV / 16; ++kk) {
+          if (pass && kk == Cfg::BKV / 16 - Cfg::HANDOVER) mbar_arrive(pass);
           // keys 16kk..16kk+15: half kk/4, packed bf16 pairs at columns 8*(kk%4) of that half
           const uint64_t offb = (uint64_t)(((kk >> 2) * Cfg::VCH_BYTES + (kk & 3) * 32) >> 4);
-          umma_bf16_ts(d, a0 + (kk >> 2) * 64 + (kk & 3) * 8, bd + offb, Cfg::IDESC_O, (j > 0 || kk > 0) ? 1u : 0u);
+          umma_bf16_ts(odst, sdst + (kk >> 2) * 64 + (kk & 3) * 8, bd + offb, Cfg::IDESC_O,
+                       (j > 0 || kk > 0) ? 1u : 0u);
         }
         umma_commit(&o_done[g]);   // measured: this commit after each PV group runs faster than none
       };
       auto v_addr = [&](int st) { return smem_u32(sKV + (st % NS) * 2 * Cfg::SLOT); };
       auto k_addr = [&](int st) { return v_addr(st) + Cfg::SLOT; };
+      uint64_t* other = &tok[1 - g];
       bool ok = mbar_wait(q_full, 0, abort_flag, p.err);
       if (ok) ok = mbar_wait(&kv_full[0], 0, abort_flag, p.err);
+      if (ok && g == 1) ok = mbar_wait(&tok[1], 0, abort_flag, p.err);    // after S_A(0)
       if (ok) {
         tc_fence_after();
-        issue_s(0, k_addr(0));
-        issue_s(1, k_addr(0));
+        issue_s(k_addr(0), other);
         umma_commit(&kv_empty[0]);
       }
+      // Token phases: tok[1] completes for S_A(0), then once per group A(j); tok[0] for
+      // S_B(0), then once per group B(j) that another group A follows.  Each hand-over
+      // comes after the receiver's previous wait on its own token, so no token runs two
+      // phases ahead of its waiter and the parity tests stay unambiguous.
       for (int j = 0; ok && j < nt; ++j) {
         const int st = j + 1;
         const bool more = j + 1 < nt;
+        if (!mbar_wait(&tok[g], g == 0 ? (j & 1) : ((j + 1) & 1), abort_flag, p.err)) break;
         if (!mbar_wait(&kv_full[st % NS], (st / NS) & 1, abort_flag, p.err)) break;
-        if (!mbar_wait(&p_full[0], j & 1, abort_flag, p.err)) break;
+        if (!mbar_wait(&p_full[g], j & 1, abort_flag, p.err)) break;
         tc_fence_after();
-        issue_pv(0, v_addr(st), j);
-        if (more) issue_s(0, k_addr(st));
-        if (!mbar_wait(&p_full[1], j & 1, abort_flag, p.err)) break;
-        tc_fence_after();
-        issue_pv(1, v_addr(st), j);
-        if (more) issue_s(1, k_addr(st));
+        // the group's last MMAs hand the token over (group B only when a group A follows)
+        uint64_t* pass = (g == 0 || more) ? other : nullptr;
+        issue_pv(v_addr(st), j, more ? nullptr : pass);
+        if (more) issue_s(k_addr(st), pass);
         umma_commit(&kv_empty[st % NS]);
       }
       if (*abort_flag) {
-        umma_commit(teardown);
-        mbar_wait_teardown(teardown, 0);
+        umma_commit(&teardown[g]);
+        mbar_wait_teardown(&teardown[g], 0);
       }
     }
   } else {
