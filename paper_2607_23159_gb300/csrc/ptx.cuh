@@ -86,38 +86,6 @@ __device__ __forceinline__ bool mbar_wait_teardown(uint64_t* bar, uint32_t parit
   return true;
 }
 
-// Exchange of one float between two warps of a CTA through a 64-bit shared-memory word
-// holding (tag << 32 | value): one store publishes both, so the reader needs no fence.
-__device__ __forceinline__ void xchg_put(uint64_t* slot, float v, uint32_t tag) {
-  const uint64_t w = ((uint64_t)tag << 32) | __float_as_uint(v);
-  asm volatile("st.shared.b64 [%0], %1;" ::"r"(smem_u32(slot)), "l"(w) : "memory");
-}
-// Spin (bounded in time) until the word carries `tag`; false on timeout or abort.
-__device__ __forceinline__ bool xchg_get(const uint64_t* slot, uint32_t tag, float* out, volatile int* abort,
-                                         int* err) {
-  const uint32_t a = smem_u32(slot);
-  uint64_t t0 = 0;
-  for (uint32_t i = 0;; ++i) {
-    uint64_t w;
-    asm volatile("ld.volatile.shared.b64 %0, [%1];" : "=l"(w) : "r"(a) : "memory");
-    if ((uint32_t)(w >> 32) == tag) {
-      *out = __uint_as_float((uint32_t)w);
-      return true;
-    }
-    if ((i & 255) == 255) {
-      if (*abort) return false;
-      const uint64_t now = globaltimer_ns();
-      if (t0 == 0) {
-        t0 = now;
-      } else if (now - t0 > CS_WAIT_TIMEOUT_NS) {
-        *abort = 1;
-        record_error(err, kErrTimeout);
-        return false;
-      }
-    }
-  }
-}
-
 // ---------------------------------------------------------------------- TMA --
 __device__ __forceinline__ void tma_prefetch_desc(const void* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");
