@@ -92,14 +92,17 @@ def test_gemm_qkv_scatter_layout(B, hd, heads, L, nb):
 
 # -------------------------------------------------------------- attention ----
 
-def _attn_case(B, hd, heads, nb, Lq, Lk, kv_shared, qscale, seed):
+def _attn_case(B, hd, heads, nb, Lq, Lk, kv_shared, qscale, seed, kramp=0.0):
     hds = max(hd, 64)
     Lks = (Lk + 7) // 8 * 8
     nkv = heads if kv_shared else nb * heads
     q = np.zeros((nb * heads, Lq, hds), np.float32)
     k = np.zeros((nkv, Lk, hds), np.float32)
     q[:, :, :hd] = bf(synth.normal(seed, (nb * heads, Lq, hd)) * qscale)
-    k[:, :, :hd] = bf(synth.normal(seed + 1, (nkv, Lk, hd)))
+    # kramp > 0 scales the keys up along the sequence, so that the running row max keeps
+    # growing from tile to tile and the lazy O rescale fires on most tiles
+    kscale = 1.0 + kramp * np.arange(Lk, dtype=np.float32)[None, :, None] / max(Lk, 1)
+    k[:, :, :hd] = bf(synth.normal(seed + 1, (nkv, Lk, hd)) * kscale)
     v = bf(synth.normal(seed + 2, (nkv, Lk, hd)))
     vt = np.zeros((nkv, hd, Lks), np.float32)
     vt[:, :, :Lk] = v.transpose(0, 2, 1)
@@ -119,6 +122,8 @@ def _attn_case(B, hd, heads, nb, Lq, Lk, kv_shared, qscale, seed):
     (128, 3, 2, 130, 512, True, 1.0),      # cross-attention: K/V shared by all batch items
     (32, 4, 4, 48, 48, False, 1.0),        # tiny model shape (one partial tile)
     (32, 4, 2, 48, 16, True, 2.0),         # tiny cross-attention, 16 text tokens
+    (128, 2, 1, 1, 129, False, 1.0),       # one query row; the last key tile holds one key
+    (128, 2, 2, 256, 1, False, 1.0),       # a single key: one tile, one valid column
 ])
 def test_attention_matches_oracle(B, hd, heads, nb, Lq, Lk, kv_shared, qscale):
     q, k, v, got = _attn_case(B, hd, heads, nb, Lq, Lk, kv_shared, qscale, seed=hd + Lq + Lk)
@@ -128,6 +133,22 @@ def test_attention_matches_oracle(B, hd, heads, nb, Lq, Lk, kv_shared, qscale):
             ref = O.attention(q[bh, :, :hd].astype(np.float64), k[bkv, :, :hd], v[bkv])
             np.testing.assert_allclose(got[j, :, h * hd:(h + 1) * hd], ref, rtol=0,
                                        atol=1e-2 * np.abs(ref).max() + 1e-3)
+
+
+@pytest.mark.parametrize("hd,Lk,kramp", [(128, 1536, 24.0), (32, 700, 30.0)])
+def test_attention_growing_row_max_rescales_match_oracle(B, hd, Lk, kramp):
+    """Keys grow along the sequence, so the running max of every row rises by more than the
+    lazy-rescale threshold on many key tiles: O and the row sums are rescaled repeatedly."""
+    heads, nb, Lq = 2, 1, 300
+    q, k, v, got = _attn_case(B, hd, heads, nb, Lq, Lk, False, 2.0, seed=17 + Lk, kramp=kramp)
+    for h in range(heads):
+        qq, kk = q[h, :, :hd].astype(np.float64), k[h, :, :hd].astype(np.float64)
+        s = qq @ kk.T / np.sqrt(hd) * np.log2(np.e)
+        tiles = s.reshape(Lq, -1)[:, :(Lk // 128) * 128].reshape(Lq, -1, 128).max(axis=2)
+        rises = (np.diff(np.maximum.accumulate(tiles, axis=1), axis=1) > 8).sum(axis=1)
+        assert rises.mean() > 2      # the case does exercise repeated rescales
+        ref = O.attention(qq, kk, v[h])
+        np.testing.assert_allclose(got[0, :, h * hd:(h + 1) * hd], ref, rtol=0, atol=1e-2 * np.abs(ref).max() + 1e-3)
 
 
 # -------------------------------------------------------------- layernorm ----
