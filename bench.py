@@ -45,6 +45,9 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", default="wan1.3b-best-of-4")
     ap.add_argument("--tau", type=float, default=None)
+    ap.add_argument("--mask", default="rule", choices=["rule", "paper-density"],
+                    help="rule: the cache rule decides; paper-density: every candidate computes on a fixed "
+                         "schedule with the skip count the paper reports (26 of 50 steps skipped)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -235,6 +238,20 @@ def run_reference(args, cfg):
 
 # ------------------------------------------------------------------ ours ----
 
+def paper_density_plan(T, K_w, K_c, skipped=None):
+    """Compute/skip plan with the paper's skip density (26 of 50 steps skipped at T = 50):
+    the K_w warm-up and K_c cool-down steps compute, and the remaining computes are spread
+    evenly over the free steps.  Returns a list of T booleans (True = compute)."""
+    skipped = round(T * 26 / 50) if skipped is None else skipped
+    free = list(range(K_w + 1, T - K_c + 1))
+    n_comp = max(0, len(free) - skipped)
+    plan = [k <= K_w or k > T - K_c for k in range(1, T + 1)]
+    for i, k in enumerate(free):
+        if (i + 1) * n_comp // len(free) > i * n_comp // len(free):
+            plan[k - 1] = True
+    return plan
+
+
 def run_ours(args, cfg):
     import torch
     rank, world, local = dist_setup(args.gpus)
@@ -254,6 +271,9 @@ def run_ours(args, cfg):
     noise = ([torch.from_numpy(synth.beam_noise(m, r, cfg.beam_keep, cfg.beam_children).reshape(-1, m.D)).cuda()
               for r in range((T - 1) // cfg.beam_every)] if beam else None)
     rnd = [0]
+    plan = paper_density_plan(T, cfg.K_w, cfg.K_c) if args.mask == "paper-density" else None
+    force_on = torch.ones(N, dtype=torch.uint8, device="cuda")
+    force_off = torch.zeros(N, dtype=torch.uint8, device="cuda")
 
     def step(i):
         """search step k = i % T + 1 of the current search (a new search every T steps);
@@ -264,7 +284,8 @@ def run_ours(args, cfg):
             rnd[0] = 0
         last = k == T
         rescore = beam and k % cfg.beam_every == 0 and not last
-        n = srch.step(k, T, tau, cfg.K_w, cfg.K_c, score=last or rescore)
+        force = None if plan is None else (force_on if plan[k - 1] else force_off)[:srch.n]
+        n = srch.step(k, T, tau, cfg.K_w, cfg.K_c, score=last or rescore, force=force)
         if rescore:
             srch.refill(srch.select(cfg.beam_keep).clone(), cfg.beam_children, cfg.beam_sigma, noise[rnd[0]])
             rnd[0] += 1
@@ -299,7 +320,7 @@ def run_ours(args, cfg):
     # end to end through the host-buffer entry point (pinned host latents in, latents + mask out)
     e2e = None
     tgrid = S.time_grid(T)
-    if not args.no_e2e and not beam:   # host-buffer path: plain best-of-N steps
+    if not args.no_e2e and not beam and args.mask == "rule":   # host-buffer path: plain best-of-N steps
         xh = torch.from_numpy(x1.copy()).pin_memory()
         skip_h = torch.zeros(N, dtype=torch.uint8).pin_memory()
         st = B.new_state(N, m.D)
@@ -342,6 +363,7 @@ def run_ours(args, cfg):
         "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded random-init weights and N(0,1) inputs)",
         "config": {"workload": cfg.name, "N": N, "T": T, "tau": tau, "K_w": cfg.K_w, "K_c": cfg.K_c,
+                   "mask": args.mask,
                    "tokens": m.L, "blocks": m.blocks, "d": m.d, "parallelism": "replicas" if world > 1 else "none",
                    "l2": f"inputs larger than L2 ({2 * synth.param_count(m) / 1e9:.1f} GB bf16 weights, GBs of activations per step)"},
         "roofline": {"kernel": "self-attention (tcgen05 flash attention)", "bound": "tensor", "achieved": ach,
