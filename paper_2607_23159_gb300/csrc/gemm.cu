@@ -10,12 +10,25 @@
 // Two TMEM accumulators (2 x BN columns) let the epilogue of tile i overlap the main
 // loop of tile i+1.  Tiles are visited n-fastest so that the CTAs in flight share A
 // rows and the whole of B in L2.
+//
+// BN = 256 runs as clusters of two CTAs on vertically adjacent tiles with the same B tile.
+// MODE 2 (the default): rank 0 issues one M = 256 tcgen05.mma (cta_group::2) per K slice for
+// the pair; each CTA's shared memory holds its 128 A rows and half of the B tile, both
+// CTAs' TMA loads complete on rank 0's stage barrier, and the MMA commit releases the stage
+// in both CTAs.  MODE 1 keeps one MMA stream per CTA and multicasts each half of B to both.
+// Measured on GB300 (M 131040): the shared-memory writes of the B tile were the limit of
+// the single-CTA kernel; MODE 2 halves them (1.66 -> 1.83 PFLOP/s at N 8960, K 1536).
+// Every output element keeps the same K order in all modes.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
 #include "common.cuh"
 #include "ptx.cuh"
 #include "tma_host.h"
+
+#ifndef CS_GEMM_PAIR_MODE
+#define CS_GEMM_PAIR_MODE 2   // the N >= 512 GEMMs: 1 = B multicast, 2 = two-SM MMA
+#endif
 
 namespace cs {
 
@@ -34,17 +47,21 @@ struct GemmArgs {
   int* err;
 };
 
-template <int BN>
+// MODE 0: one CTA per tile.  MODE 1: clusters of two, B multicast.  MODE 2: clusters of
+// two running one M = 256 tcgen05.mma (cta_group::2) per K slice: each CTA holds its 128 A
+// rows and half of the B tile, so every stage is half as large and the ring deeper.
+template <int BN, int MODE = 0>
 struct GemmCfg {
   static constexpr int BM = 128, BK = 64;
-  static constexpr int STAGES = BN == 256 ? 4 : 6;
+  static constexpr int B_ROWS = MODE == 2 ? BN / 2 : BN;   // B rows held in this CTA's shared memory
+  static constexpr int STAGES = MODE == 2 ? 6 : (BN == 256 ? 4 : 6);
   static constexpr int A_BYTES = BM * BK * 2;
-  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int B_BYTES = B_ROWS * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int TMEM_COLS = 2 * BN;
   static constexpr int OUT_BYTES = 4 * 2 * 32 * 128;   // per epilogue warp: two 32 x 32 float32 staging buffers
   static constexpr int SMEM = STAGES * STAGE_BYTES + OUT_BYTES + 1024 + 256;
-  static constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
+  static constexpr uint32_t IDESC = idesc_bf16_f32(MODE == 2 ? 2 * BM : BM, BN);
 };
 
 // tanh on the SFU (tanh.approx.f32: the hardware instruction, relative error ~2^-11, below
@@ -151,11 +168,13 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& p, int m, int n, 
   }
 }
 
-template <int BN, int EPI>
+template <int BN, int EPI, int MODE>
 __global__ void __launch_bounds__(192, 1)
     gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmC, const GemmArgs p) {
-  using Cfg = GemmCfg<BN>;
+  using Cfg = GemmCfg<BN, MODE>;
+  constexpr bool PAIR = MODE != 0;     // clusters of two CTAs on vertically adjacent tiles
+  constexpr bool TWO_SM = MODE == 2;   // one cta_group::2 MMA stream issued by the cluster's rank 0
   constexpr int BM = Cfg::BM, BK = Cfg::BK, STAGES = Cfg::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -174,28 +193,42 @@ __global__ void __launch_bounds__(192, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], MODE == 1 ? 2 : 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 4);
+      mbar_init(&tempty[a], TWO_SM ? 8 : 4);   // TWO_SM: rank 0's barrier, both CTAs' epilogue warps
     }
     mbar_init(teardown, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
-    tmem_relinquish();
+    if constexpr (TWO_SM) {
+      tmem_alloc_2sm(tmem_slot, Cfg::TMEM_COLS);   // collective with the peer CTA's warp 1
+      tmem_relinquish_2sm();
+    } else {
+      tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
   __syncthreads();
+  if (PAIR) cluster_sync();   // the peer's barriers exist before anything is multicast into it
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
   const int m_tiles = (p.M + BM - 1) / BM, n_tiles = (p.N + BN - 1) / BN;
-  const int tiles = m_tiles * n_tiles;
   const int kblocks = p.K / BK;
+  // work items, n-fastest: single CTA -> (m-tile, n-tile); PAIR -> (pair of m-tiles, n-tile),
+  // of which the CTA of cluster rank r takes m-tile 2 * pair + r (rows past M are zero-filled
+  // by TMA and never stored)
+  const int rank = PAIR ? (int)cluster_ctarank() : 0;
+  const int items = PAIR ? ((m_tiles + 1) / 2) * n_tiles : m_tiles * n_tiles;
+  const int first = PAIR ? (int)blockIdx.x / 2 : (int)blockIdx.x;
+  const int stride = PAIR ? (int)gridDim.x / 2 : (int)gridDim.x;
+  auto item_m0 = [&](int it) { return (PAIR ? 2 * (it / n_tiles) + rank : it / n_tiles) * BM; };
+  auto item_n0 = [&](int it) { return (it % n_tiles) * BN; };
 
   if (warp == 0) {
     if (lane == 0) {
@@ -204,18 +237,37 @@ __global__ void __launch_bounds__(192, 1)
       int stage = 0;
       uint32_t phase = 0;
       int issued = 0;
-      for (int tile = blockIdx.x; tile < tiles && !*abort_flag; tile += gridDim.x) {
-        const int m0 = (tile / n_tiles) * BM, n0 = (tile % n_tiles) * BN;
+      for (int it = first; it < items && !*abort_flag; it += stride) {
+        const int m0 = item_m0(it), n0 = item_n0(it);
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.err)) break;
-          mbar_arrive_expect_tx(&full[stage], Cfg::STAGE_BYTES);
-          tma_load_2d(sA + stage * Cfg::A_BYTES, &tmA, &full[stage], kb * BK, m0);
-          tma_load_2d(sB + stage * Cfg::B_BYTES, &tmB, &full[stage], kb * BK, n0);
+          if constexpr (TWO_SM) {
+            // both CTAs' halves complete on rank 0's barrier, which rank 0 arms for all of them
+            if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * Cfg::STAGE_BYTES);
+            const uint32_t bar0 = cluster_map(&full[stage], 0);
+            tma_load_2d_2sm(sA + stage * Cfg::A_BYTES, &tmA, bar0, kb * BK, m0);
+            tma_load_2d_2sm(sB + stage * Cfg::B_BYTES, &tmB, bar0, kb * BK, n0 + rank * (BN / 2));
+          } else {
+            mbar_arrive_expect_tx(&full[stage], Cfg::STAGE_BYTES);   // MODE 1: half of B comes from the peer
+            tma_load_2d(sA + stage * Cfg::A_BYTES, &tmA, &full[stage], kb * BK, m0);
+            if (PAIR)
+              tma_load_2d_mc(sB + stage * Cfg::B_BYTES + rank * (Cfg::B_BYTES / 2), &tmB, &full[stage], kb * BK,
+                             n0 + rank * (BN / 2), 0x3);
+            else
+              tma_load_2d(sB + stage * Cfg::B_BYTES, &tmB, &full[stage], kb * BK, n0);
+          }
           ++issued;
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
         }
       }
-      if (*abort_flag) {
+      if (PAIR && !*abort_flag) {
+        // every stage released by both CTAs' MMAs: no arrival from the peer is still on its way
+        for (int i = 0; i < STAGES; ++i) {
+          mbar_wait_teardown(&empty[stage], phase ^ 1);
+          if (++stage == STAGES) { stage = 0; phase ^= 1; }
+        }
+      }
+      if (*abort_flag && !(TWO_SM && rank != 0)) {
         // drain: wait (bounded) for the loads of the last ring's worth of stages
         for (int back = 1; back <= STAGES && back <= issued; ++back) {
           int s = stage - back, ph = phase;
@@ -225,13 +277,14 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && !(TWO_SM && rank != 0)) {   // TWO_SM: rank 0 issues for the pair
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
       uint32_t acc_phase = 0;
-      for (int tile = blockIdx.x; tile < tiles && !*abort_flag; tile += gridDim.x) {
+      for (int it = first; it < items && !*abort_flag; it += stride) {
         if (!mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.err)) break;
+        if constexpr (TWO_SM) fence_acq_rel_cluster();   // the peer's epilogue arrived from another CTA
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
         bool ok = true;
@@ -242,19 +295,27 @@ __global__ void __launch_bounds__(192, 1)
           const uint32_t b0 = smem_u32(sB + stage * Cfg::B_BYTES);
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
-            umma_bf16_ss(d_tmem, sdesc_sw128(a0 + k * 32), sdesc_sw128(b0 + k * 32), Cfg::IDESC,
-                         (kb | k) != 0 ? 1u : 0u);
-          umma_commit(&empty[stage]);
+            if constexpr (TWO_SM)
+              umma_bf16_ss_2sm(d_tmem, sdesc_sw128(a0 + k * 32), sdesc_sw128(b0 + k * 32), Cfg::IDESC,
+                               (kb | k) != 0 ? 1u : 0u);
+            else
+              umma_bf16_ss(d_tmem, sdesc_sw128(a0 + k * 32), sdesc_sw128(b0 + k * 32), Cfg::IDESC,
+                           (kb | k) != 0 ? 1u : 0u);
+          if constexpr (TWO_SM) umma_commit_2sm_mc(&empty[stage], 0x3);
+          else if constexpr (PAIR) umma_commit_mc(&empty[stage], 0x3);
+          else umma_commit(&empty[stage]);
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
         }
         if (!ok) break;
-        umma_commit(&tfull[acc]);
+        if constexpr (TWO_SM) umma_commit_2sm_mc(&tfull[acc], 0x3);   // both CTAs' accumulators
+        else umma_commit(&tfull[acc]);
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1;
       }
       if (*abort_flag) {
         // every MMA issued so far must finish before TMEM is released
-        umma_commit(teardown);
+        if constexpr (TWO_SM) umma_commit_2sm_mc(teardown, 0x1);
+        else umma_commit(teardown);
         mbar_wait_teardown(teardown, 0);
       }
     }
@@ -265,11 +326,12 @@ __global__ void __launch_bounds__(192, 1)
     uint32_t acc_phase = 0;
     int nout = 0;   // chunks this warp has handed to TMA
     if (lane == 0 && p.tma_out) tma_prefetch_desc(&tmC);
-    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+    for (int it = first; it < items; it += stride) {
       if (!__all_sync(0xffffffffu, mbar_wait(&tfull[acc], acc_phase, abort_flag, p.err))) break;
       tc_fence_after();
-      const int m0 = (tile / n_tiles) * BM, n0 = (tile % n_tiles) * BN;
+      const int m0 = item_m0(it), n0 = item_n0(it);
       const int m = m0 + row;
+      const bool rows_in = m0 + sp * 32 < p.M;   // this warp has rows to store (uniform)
       const uint32_t tbase = tmem_base + ((uint32_t)(sp * 32) << 16) + acc * BN;
       if constexpr (EPI == CS_EPI_BF16 || EPI == CS_EPI_GELU_BF16) {
         if (p.tma_out) {
@@ -277,7 +339,7 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll 1
           for (int c = 0; c < BN / 64; ++c) {
             const int n = n0 + c * 64;
-            if (n >= p.N) break;   // uniform across the warp
+            if (n >= p.N || !rows_in) break;   // uniform across the warp
             uint32_t r0[32], r1[32];
             tmem_ld32(tbase + c * 64, r0);
             tmem_ld32(tbase + c * 64 + 32, r1);
@@ -316,7 +378,10 @@ __global__ void __launch_bounds__(192, 1)
           }
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive(&tempty[acc]);
+          if (lane == 0) {
+            if (TWO_SM) mbar_arrive_cluster(cluster_map(&tempty[acc], 0));
+            else mbar_arrive(&tempty[acc]);
+          }
           acc ^= 1;
           if (acc == 0) acc_phase ^= 1;
           continue;
@@ -330,6 +395,7 @@ __global__ void __launch_bounds__(192, 1)
         tmem_ld32(tbase + c * 32, r);
         if constexpr (EPI == CS_EPI_F32 || EPI == CS_EPI_RESID_F32) {
           if (p.tma_out) {
+            if (!rows_in) continue;
             // this warp's 32 rows x 32 columns -> 128-byte-swizzled staging -> one TMA op
             // (a plain store, or for the residual an add performed in L2)
             uint8_t* buf = sOut + (sp * 2 + (nout & 1)) * 4096;
@@ -369,7 +435,10 @@ __global__ void __launch_bounds__(192, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[acc]);
+      if (lane == 0) {
+        if (TWO_SM) mbar_arrive_cluster(cluster_map(&tempty[acc], 0));
+        else mbar_arrive(&tempty[acc]);
+      }
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1;
     }
@@ -378,22 +447,25 @@ __global__ void __launch_bounds__(192, 1)
 
   tc_fence_before();
   __syncthreads();
+  if (PAIR) cluster_sync();   // the peer has consumed everything this CTA multicast to it
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
+    if constexpr (TWO_SM) tmem_dealloc_2sm(tmem_base, Cfg::TMEM_COLS);
+    else tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
   }
 }
 
-template <int BN, int EPI>
+template <int BN, int EPI, int MODE>
 static cs_status launch_gemm(const void* A, const void* B, const GemmArgs& args, cudaStream_t stream) {
-  using Cfg = GemmCfg<BN>;
+  using Cfg = GemmCfg<BN, MODE>;
+  constexpr bool PAIR = MODE != 0;
   CUtensorMap ta, tb;
   const uint64_t da[2] = {(uint64_t)args.K, (uint64_t)args.M};
   const uint64_t sa[1] = {(uint64_t)args.K * 2};
   const uint32_t ba[2] = {64, 128};
   CS_TRY(make_tmap_bf16(&ta, A, 2, da, sa, ba));
   const uint64_t db[2] = {(uint64_t)args.K, (uint64_t)args.N};
-  const uint32_t bb[2] = {64, (uint32_t)BN};
+  const uint32_t bb[2] = {64, (uint32_t)(PAIR ? BN / 2 : BN)};   // PAIR: each CTA loads half of the B tile
   CS_TRY(make_tmap_bf16(&tb, B, 2, db, sa, bb));
   // float32 outputs go through TMA when the output rows are TMA-addressable
   GemmArgs a = args;
@@ -415,19 +487,44 @@ static cs_status launch_gemm(const void* A, const void* B, const GemmArgs& args,
     CS_TRY(make_tmap(&tc, args.out, 2, dc, sc, bc, false));
     a.tma_out = 1;
   }
-  auto kern = gemm_tcgen05_kernel<BN, EPI>;
+  auto kern = gemm_tcgen05_kernel<BN, EPI, MODE>;
   CS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
-  const int tiles = ((args.M + 127) / 128) * ((args.N + BN - 1) / BN);
-  const int grid = tiles < num_sms() ? tiles : num_sms();
-  kern<<<grid, 192, Cfg::SMEM, stream>>>(ta, tb, tc, a);
+  const int m_tiles = (args.M + 127) / 128, n_tiles = (args.N + BN - 1) / BN;
+  if (!PAIR) {
+    const int tiles = m_tiles * n_tiles;
+    const int grid = tiles < num_sms() ? tiles : num_sms();
+    kern<<<grid, 192, Cfg::SMEM, stream>>>(ta, tb, tc, a);
+    CS_LAUNCHED();
+    return CS_OK;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(192);
+  cfg.dynamicSmemBytes = Cfg::SMEM;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cfg.gridDim = dim3(num_sms() / 2 * 2);
+  static int max_clusters = 0;   // co-resident clusters of two (one CTA per SM)
+  if (max_clusters == 0) {
+    CS_CUDA(cudaOccupancyMaxActiveClusters(&max_clusters, kern, &cfg));
+    CS_REQUIRE(max_clusters > 0, "gemm: no cluster of two CTAs fits on this device");
+  }
+  const int items = ((m_tiles + 1) / 2) * n_tiles;
+  cfg.gridDim = dim3(2 * (items < max_clusters ? items : max_clusters));
+  CS_CUDA(cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, a));
   CS_LAUNCHED();
   return CS_OK;
 }
 
 template <int EPI>
 static cs_status dispatch_bn(const void* A, const void* B, const GemmArgs& args, cudaStream_t stream) {
-  if (args.N >= 512) return launch_gemm<256, EPI>(A, B, args, stream);
-  return launch_gemm<128, EPI>(A, B, args, stream);
+  if (args.N >= 512) return launch_gemm<256, EPI, CS_GEMM_PAIR_MODE>(A, B, args, stream);
+  return launch_gemm<128, EPI, 0>(A, B, args, stream);
 }
 
 cs_status gemm_run(const void* A, const void* B, int epi, const GemmArgs& args, cudaStream_t stream) {
