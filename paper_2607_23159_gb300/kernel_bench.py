@@ -6,6 +6,10 @@
 
 Inputs are random device tensors (the timing does not depend on their values).  Prints
 one JSON line with the average launch time and the achieved TFLOP/s or GB/s.
+
+``--torch`` times PyTorch's own kernels on the same shape instead (informal comparators,
+never part of the library's path): ``scaled_dot_product_attention`` for attention,
+``torch.matmul`` for the GEMMs, and the cache step written as torch elementwise ops.
 """
 from __future__ import annotations
 
@@ -47,11 +51,41 @@ def main():
     ap.add_argument("--skip-frac", type=float, default=1.0)
     ap.add_argument("--reps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=2)
+    ap.add_argument("--torch", action="store_true", help="time the PyTorch comparator instead")
     a = ap.parse_args()
     dev = "cuda"
     bf = torch.bfloat16
-    out = {"kernel": a.kernel}
-    if a.kernel == "attention":
+    out = {"kernel": a.kernel, "impl": "torch" if a.torch else "ours"}
+    if a.torch and a.kernel == "attention":
+        Lk = a.Lk or a.L
+        q = torch.randn(a.batch, a.heads, a.L, a.hd, device=dev).to(bf)
+        k = torch.randn(a.batch, a.heads, Lk, a.hd, device=dev).to(bf)
+        v = torch.randn(a.batch, a.heads, Lk, a.hd, device=dev).to(bf)
+        sdpa = torch.nn.functional.scaled_dot_product_attention
+        ms = _time(lambda: sdpa(q, k, v), a.reps, a.warmup)
+        out.update(shape=dict(batch=a.batch, L=a.L, Lk=Lk, heads=a.heads, hd=a.hd), ms=ms,
+                   tflops=4.0 * a.batch * a.heads * a.L * Lk * a.hd / (ms / 1e3) / 1e12)
+    elif a.torch and a.kernel in ("gemm", "qkv"):
+        N = a.N if a.kernel == "gemm" else 3 * a.heads * a.hd
+        M = a.M if a.kernel == "gemm" else a.batch * a.L
+        A = torch.randn(M, a.K, device=dev).to(bf)
+        W = (torch.randn(N, a.K, device=dev) * 0.05).to(bf)
+        ms = _time(lambda: torch.matmul(A, W.t()), a.reps, a.warmup)
+        out.update(shape=dict(M=M, N=N, K=a.K), ms=ms, tflops=2.0 * M * N * a.K / (ms / 1e3) / 1e12)
+    elif a.torch and a.kernel in ("cache", "cache-fused"):
+        N, D = a.N, a.D
+        x = torch.randn(N, D, device=dev)
+        xr = x * 0.99
+        delta = torch.randn(N, D, device=dev)
+        h = -0.02
+
+        def run():   # every candidate skipped: drift, then x += h (x + delta)
+            d = torch.linalg.vector_norm(x - xr, dim=1) / torch.linalg.vector_norm(xr, dim=1)
+            x.add_(x + delta, alpha=h)
+            return d
+        ms = _time(run, a.reps, a.warmup)
+        out.update(shape=dict(N=N, D=D, skipped=N), ms=ms, gbs=16.0 * N * D / (ms / 1e3) / 1e9)
+    elif a.kernel == "attention":
         Lk = a.Lk or a.L
         hds = max(a.hd, 64)
         BH = a.batch * a.heads
