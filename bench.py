@@ -45,6 +45,10 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", default="wan1.3b-best-of-4")
     ap.add_argument("--tau", type=float, default=None)
+    ap.add_argument("--search", default="best-of-n", choices=["best-of-n", "pruned", "static", "commit", "cfg"],
+                    help="best-of-n (or the config's beam): the default; pruned: prune to the top half at "
+                         "0.4 T and finish; static: fixed every-3rd-step schedule; commit: the winner's seed "
+                         "alone at tau = 0; cfg: guided search (w = 5, one cache state per branch)")
     ap.add_argument("--mask", default="rule", choices=["rule", "paper-density"],
                     help="rule: the cache rule decides; paper-density: every candidate computes on a fixed "
                          "schedule with the skip count the paper reports (26 of 50 steps skipped)")
@@ -261,9 +265,15 @@ def run_ours(args, cfg):
     tau = cfg.tau if args.tau is None else args.tau
     x1 = synth.initial_noise(m, range(N)).reshape(N, -1)
     y = synth.target_latent(m).reshape(-1)
-    model = B.Model(m, N)
+    mode = args.search
+    if mode == "commit":           # Algorithm 1's commit: the winner's seed alone at full compute
+        N, tau = 1, 0.0
+        x1 = x1[:1]
+    model = B.Model(m, 2 * N if mode == "cfg" else N)
     model.load_streamed()          # seeded weights generated and loaded tensor by tensor
     model.set_text_context(torch.from_numpy(synth.text_context(m)).cuda())
+    if mode == "cfg":
+        model.set_null_text_context(torch.zeros(m.Lt, m.d_text, device="cuda"))
     x1_dev = torch.from_numpy(x1).cuda()
     y_dev = torch.from_numpy(y).cuda()
     srch = S.Search(model, N, target=y_dev)
@@ -274,24 +284,44 @@ def run_ours(args, cfg):
     plan = paper_density_plan(T, cfg.K_w, cfg.K_c) if args.mask == "paper-density" else None
     force_on = torch.ones(N, dtype=torch.uint8, device="cuda")
     force_off = torch.zeros(N, dtype=torch.uint8, device="cuda")
+    prune_step, prune_keep = max(1, round(0.4 * T)), max(1, N // 2)
+    tgrid_f = S.time_grid(T)
+    if mode == "cfg":
+        st_cfg = B.new_state_cfg(N, m.D)
+        skip_cfg = torch.zeros(2 * N, dtype=torch.uint8, device="cuda")
+        scores_cfg = torch.zeros(N, device="cuda")
 
     def step(i):
         """search step k = i % T + 1 of the current search (a new search every T steps);
-        beam workloads rescore and refill every beam_every steps."""
+        beam workloads rescore and refill every beam_every steps.  Returns (computed DiT
+        items, candidates advanced)."""
         k = i % T + 1
+        last = k == T
+        if mode == "cfg":
+            if k == 1:
+                st_cfg["x"].copy_(x1_dev)
+                st_cfg["has_ref"].zero_()
+                st_cfg["accum"].zero_()
+            n = model.search_step_cfg(st_cfg, k, T, float(tgrid_f[k - 1]), float(tgrid_f[k]), tau, cfg.K_w, cfg.K_c,
+                                      5.0, skip_cfg, target=y_dev if last else None, scores=scores_cfg if last else None)
+            return n, N
         if k == 1:
             srch.reset(x1_dev)
             rnd[0] = 0
-        last = k == T
+        advanced = srch.n
         rescore = beam and k % cfg.beam_every == 0 and not last
+        prune = mode == "pruned" and k == prune_step
         force = None if plan is None else (force_on if plan[k - 1] else force_off)[:srch.n]
-        n = srch.step(k, T, tau, cfg.K_w, cfg.K_c, score=last or rescore, force=force)
+        n = srch.step(k, T, tau, cfg.K_w, cfg.K_c, score=last or rescore or prune, force=force,
+                      schedule_every=3 if mode == "static" else 0)
         if rescore:
             srch.refill(srch.select(cfg.beam_keep).clone(), cfg.beam_children, cfg.beam_sigma, noise[rnd[0]])
             rnd[0] += 1
+        if prune:
+            srch.refill(srch.select(prune_keep).clone(), 0, 0.0, None)
         if last:
             srch.select(1)
-        return n
+        return n, advanced
 
     for i in range(args.warmup):
         step(i)
@@ -300,13 +330,16 @@ def run_ours(args, cfg):
     model.set_profiling(True)
     launches0 = B.launch_count()
     computed = 0
+    advanced = 0
     barrier(world)
     torch.cuda.synchronize()
     with ClockSampler(local) as clk:
         ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         ev0.record()
         for i in range(args.steps):
-            computed += step(i)
+            c, a = step(i)
+            computed += c
+            advanced += a
         ev1.record()
         torch.cuda.synchronize()
         barrier(world)
@@ -315,12 +348,12 @@ def run_ours(args, cfg):
     model.set_profiling(False)
     stats = {c: model.kernel_stats(c) for c in range(5)}
     ms = max_over_ranks(ms_local, world)
-    value = job_throughput(N * args.steps, ms_local / 1e3, world)
+    value = job_throughput(advanced, ms_local / 1e3, world)
 
     # end to end through the host-buffer entry point (pinned host latents in, latents + mask out)
     e2e = None
     tgrid = S.time_grid(T)
-    if not args.no_e2e and not beam and args.mask == "rule":   # host-buffer path: plain best-of-N steps
+    if not args.no_e2e and not beam and args.mask == "rule" and mode == "best-of-n":   # host-buffer path
         xh = torch.from_numpy(x1.copy()).pin_memory()
         skip_h = torch.zeros(N, dtype=torch.uint8).pin_memory()
         st = B.new_state(N, m.D)
@@ -362,7 +395,7 @@ def run_ours(args, cfg):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded random-init weights and N(0,1) inputs)",
-        "config": {"workload": cfg.name, "N": N, "T": T, "tau": tau, "K_w": cfg.K_w, "K_c": cfg.K_c,
+        "config": {"workload": cfg.name, "N": N, "T": T, "tau": tau, "K_w": cfg.K_w, "K_c": cfg.K_c, "search": mode,
                    "mask": args.mask,
                    "tokens": m.L, "blocks": m.blocks, "d": m.d, "parallelism": "replicas" if world > 1 else "none",
                    "l2": f"inputs larger than L2 ({2 * synth.param_count(m) / 1e9:.1f} GB bf16 weights, GBs of activations per step)"},
@@ -377,7 +410,7 @@ def run_ours(args, cfg):
             "cache_update": {"launches": n_c, "ms": ms_c, "gbs": cache_gbs, "frac_hbm": cache_gbs / hbm},
             "other": {"launches": stats[B.KC_OTHER][0], "ms": stats[B.KC_OTHER][1]},
         },
-        "computed_fraction": computed / (N * args.steps),
+        "computed_fraction": computed / ((2 if mode == "cfg" else 1) * advanced),
         "gpu_launches": launches,
         "clocks": clk.summary(),
     }
