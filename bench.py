@@ -213,6 +213,19 @@ def cpu_baseline(cfg, rows=512):
                        f"candidate-step counted as computed (skipped steps cost the oracle ~1000x less)")}
 
 
+def workload_config(args, cfg):
+    """The `config` object of the JSON line (the same for both arms)."""
+    from paper_2607_23159_gb300 import synth
+    m = cfg.model
+    commit = args.search == "commit"
+    return {"workload": cfg.name, "N": 1 if commit else cfg.N, "T": cfg.T,
+            "tau": 0.0 if commit else (cfg.tau if args.tau is None else args.tau), "K_w": cfg.K_w, "K_c": cfg.K_c,
+            "search": args.search, "mask": args.mask, "tokens": m.L, "blocks": m.blocks, "d": m.d,
+            "parallelism": "replicas" if args.gpus > 1 else "none",
+            "l2": f"inputs larger than L2 ({2 * synth.param_count(m) / 1e9:.1f} GB bf16 weights, GBs of "
+                  f"activations per step)"}
+
+
 def run_reference(args, cfg):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -230,7 +243,7 @@ def run_reference(args, cfg):
     line = {"impl": "reference", "metric": METRIC, "value": val, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * cfg.N / val, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": cfg.name, "N": cfg.N, "T": cfg.T, "tau": cfg.tau},
+            "config": workload_config(args, cfg),
             "cpu_baseline": {"value": val, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                              "sample": (f"per step: fp64 numpy oracle on one block, K/V of "
                                         f"{min(2048, cfg.model.L)} and query rows {min(128, cfg.model.L)} of "
@@ -395,10 +408,7 @@ def run_ours(args, cfg):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded random-init weights and N(0,1) inputs)",
-        "config": {"workload": cfg.name, "N": N, "T": T, "tau": tau, "K_w": cfg.K_w, "K_c": cfg.K_c, "search": mode,
-                   "mask": args.mask,
-                   "tokens": m.L, "blocks": m.blocks, "d": m.d, "parallelism": "replicas" if world > 1 else "none",
-                   "l2": f"inputs larger than L2 ({2 * synth.param_count(m) / 1e9:.1f} GB bf16 weights, GBs of activations per step)"},
+        "config": workload_config(args, cfg),
         "roofline": {"kernel": "self-attention (tcgen05 flash attention)", "bound": "tensor", "achieved": ach,
                      "peak": peak_tf, "peak_source": peak_src, "unit": "TFLOP/s", "frac": ach / peak_tf,
                      "traffic": traffic, "launches": n_sa, "avg_ms": ms_sa / n_sa if n_sa else None},
