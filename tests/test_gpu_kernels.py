@@ -65,6 +65,30 @@ def test_gemm_epilogues_match_oracle_linear(B, M, N, K):
     assert int(err[0]) == 0
 
 
+@pytest.mark.parametrize("M,N,K", [(1, 512, 64), (129, 544, 128), (257, 520, 64), (1000, 800, 320),
+                                   (255, 1024, 64), (383, 2560, 128)])
+def test_gemm_cluster_pairs_ragged_shapes(B, M, N, K):
+    """N >= 512 runs on clusters of two CTAs (one M = 256 MMA per pair): odd tile counts leave
+    the second CTA of the last pair without rows, N tails leave half a B tile out of range, and
+    N % 32 != 0 takes the non-TMA epilogue.  float32 and residual outputs against the oracle."""
+    A = bf(synth.normal(500 + M, (M, K)))
+    W = bf(synth.normal(600 + N, (N, K)) * 0.1)
+    bias = synth.normal(700 + N, (N,))
+    ref = O.linear(A, W, bias)
+    scale = np.abs(ref).max()
+    err = err_word()
+    Ad, Wd = dev(A, torch.bfloat16), dev(W, torch.bfloat16)
+    out = torch.full((M, N), 7.0, device="cuda")
+    B.gemm(Ad, Wd, B.EPI_F32, out, bias=dev(bias), err=err)
+    np.testing.assert_allclose(out.cpu().numpy(), ref, rtol=0, atol=2e-5 * scale)
+    res0 = synth.normal(800, (M, N))
+    res = dev(res0)
+    B.gemm(Ad, Wd, B.EPI_RESID_F32, res, bias=dev(bias), gate=None, err=err)
+    np.testing.assert_allclose(res.cpu().numpy(), res0 + ref, rtol=0, atol=4e-5 * scale)
+    torch.cuda.synchronize()
+    assert int(err[0]) == 0
+
+
 @pytest.mark.parametrize("hd,heads,L,nb", [(128, 2, 200, 3), (32, 4, 48, 2)])
 def test_gemm_qkv_scatter_layout(B, hd, heads, L, nb):
     d = hd * heads
