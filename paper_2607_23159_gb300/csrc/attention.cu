@@ -114,7 +114,7 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
     tmem_relinquish();
   }
   tc_fence_before();
-  __syncthreads();
+  block_sync();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -324,7 +324,7 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
   }
 
   tc_fence_before();
-  __syncthreads();
+  block_sync();
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, 512);

@@ -41,7 +41,7 @@ __device__ __forceinline__ void block_sum(float (&v)[NV], float (*red)[32]) {
 #pragma unroll
     for (int q = 0; q < NV; ++q) red[q][warp] = v[q];
   }
-  __syncthreads();
+  block_sync();
   if (warp == 0) {
     const int nw = blockDim.x >> 5;
 #pragma unroll
@@ -184,7 +184,7 @@ __global__ void decide_finalize_kernel(const float* __restrict__ partials, int n
       flags[i] = compute ? 1 : 0;
     }
   }
-  __syncthreads();
+  block_sync();
   if (threadIdx.x == 0) {
     int n = 0;
     for (int i = 0; i < N; ++i)
@@ -366,7 +366,7 @@ __global__ void score_finalize_kernel(const float* __restrict__ partials, int nc
 // Grid-wide barrier over co-resident CTAs (cooperative launch), bounded in time.
 // bar[0] counts arrivals, bar[1] is the generation; bar[0] must be 0 at launch.
 __device__ __forceinline__ void grid_barrier(unsigned* bar, int* err) {
-  __syncthreads();
+  block_sync();
   if (threadIdx.x == 0) {
     volatile unsigned* gen = bar + 1;
     const unsigned g = *gen;
@@ -387,7 +387,7 @@ __device__ __forceinline__ void grid_barrier(unsigned* bar, int* err) {
     }
     __threadfence();
   }
-  __syncthreads();
+  block_sync();
 }
 
 template <bool kScore>
@@ -412,7 +412,7 @@ __global__ void __launch_bounds__(kCacheThreads) decide_skip_kernel(
     a_s[i] = accum[i];
     had[i] = has_ref[i];
   }
-  __syncthreads();
+  block_sync();
   // (1) drift partials
   if (!wf) {
     for (int item = it0; item < it1; ++item) {
@@ -438,7 +438,7 @@ __global__ void __launch_bounds__(kCacheThreads) decide_skip_kernel(
         partials[((long long)i * nch + c) * 2 + 0] = v[0];
         partials[((long long)i * nch + c) * 2 + 1] = v[1];
       }
-      __syncthreads();
+      block_sync();
     }
   }
   // (2) every partial is written
@@ -482,7 +482,7 @@ __global__ void __launch_bounds__(kCacheThreads) decide_skip_kernel(
       }
     }
   }
-  __syncthreads();
+  block_sync();
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     int n = 0;
     for (int i = 0; i < N; ++i)
@@ -526,7 +526,7 @@ __global__ void __launch_bounds__(kCacheThreads) decide_skip_kernel(
     if (kScore) {
       block_sum<1>(acc, red);
       if (threadIdx.x == 0) spart[(long long)i * nch + c] = acc[0];
-      __syncthreads();
+      block_sync();
     }
   }
 }
@@ -573,7 +573,7 @@ __global__ void __launch_bounds__(kCacheThreads) apply_computed_kernel(
 __global__ void topk_kernel(const float* __restrict__ scores, int N, int k, int32_t* __restrict__ idx) {
   extern __shared__ float s[];
   for (int i = threadIdx.x; i < N; i += blockDim.x) s[i] = scores[i];
-  __syncthreads();
+  block_sync();
   for (int i = threadIdx.x; i < N; i += blockDim.x) {
     const float si = s[i];
     const bool ni = isnan(si);

@@ -213,7 +213,7 @@ __global__ void __launch_bounds__(192, 1)
     }
   }
   tc_fence_before();
-  __syncthreads();
+  block_sync();
   if (PAIR) cluster_sync();   // the peer's barriers exist before anything is multicast into it
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
@@ -446,7 +446,7 @@ __global__ void __launch_bounds__(192, 1)
   }
 
   tc_fence_before();
-  __syncthreads();
+  block_sync();
   if (PAIR) cluster_sync();   // the peer has consumed everything this CTA multicast to it
   if (warp == 1) {
     tc_fence_after();

@@ -21,6 +21,15 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+// CTA barrier reached by whole warps.  The kernels give one lane of a warp a role (TMA
+// producer, MMA issuer, a bulk-store drain) while the other 31 lanes go ahead to the
+// barrier; reconverging the warp first keeps the barrier a whole-warp operation.  Every
+// lane of the CTA must call this.
+__device__ __forceinline__ void block_sync() {
+  __syncwarp();
+  __syncthreads();
+}
+
 __device__ __forceinline__ uint64_t globaltimer_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
@@ -239,6 +248,7 @@ __device__ __forceinline__ uint32_t cluster_ctarank() {
 }
 // All threads of every CTA of the cluster: release/acquire rendezvous.
 __device__ __forceinline__ void cluster_sync() {
+  __syncwarp();   // the whole warp executes the .aligned barrier together
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
