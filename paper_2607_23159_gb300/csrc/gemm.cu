@@ -509,11 +509,16 @@ static cs_status launch_gemm(const void* A, const void* B, const GemmArgs& args,
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   cfg.gridDim = dim3(num_sms() / 2 * 2);
-  static int max_clusters = 0;   // co-resident clusters of two (one CTA per SM)
-  if (max_clusters == 0) {
-    CS_CUDA(cudaOccupancyMaxActiveClusters(&max_clusters, kern, &cfg));
-    CS_REQUIRE(max_clusters > 0, "gemm: no cluster of two CTAs fits on this device");
+  static int max_clusters = -1;   // co-resident clusters of two (one CTA per SM); -1 = not asked yet
+  if (max_clusters < 0) {
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+      (void)cudaGetLastError();
+      n = 0;
+    }
+    max_clusters = n;
   }
+  if (max_clusters == 0) return launch_gemm<BN, EPI, 0>(A, B, args, stream);   // no cluster fits: one CTA per tile
   const int items = ((m_tiles + 1) / 2) * n_tiles;
   cfg.gridDim = dim3(2 * (items < max_clusters ? items : max_clusters));
   CS_CUDA(cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, a));
