@@ -265,6 +265,14 @@ cs_status cs_reset_kernel_stats(cs_model* model);
 /* Kernel launches this library has issued in this process (all entry points). */
 long long cs_launch_count(void);
 
+/* Self-test of the failure path (the paper has no counterpart).  Launches one kernel
+ * whose thread waits on an mbarrier that nothing arrives on, with the bounded wait every
+ * kernel of this library uses: after CS_WAIT_TIMEOUT_NS (2 s) of GPU time the wait gives
+ * up, CS_ERR_TIMEOUT is written to *err_dev (device int, first error wins: clear it
+ * first) and the kernel returns, so the CUDA context stays usable.  Returns CS_OK once
+ * the launch is queued on `stream`, CS_ERR_ARG for a null err_dev. */
+cs_status cs_selftest_bounded_wait(int* err_dev, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -39,6 +39,7 @@ class ModelConfig(C.Structure):
 P, I, LL, F, D, SZ = C.c_void_p, C.c_int, C.c_longlong, C.c_float, C.c_double, C.c_size_t
 
 _SIGS = {
+    "cs_selftest_bounded_wait": (I, [P, P]),
     "cs_last_error": (C.c_char_p, []),
     "cs_version": (C.c_char_p, []),
     "cs_param_count": (SZ, [C.POINTER(ModelConfig)]),
@@ -331,3 +332,9 @@ def new_state(N: int, D: int, device="cuda"):
         "accum": torch.zeros(N, dtype=torch.float32, device=device),
         "has_ref": torch.zeros(N, dtype=torch.uint8, device=device),
     }
+
+
+def selftest_bounded_wait(err, stream=None):
+    """Queue the failure-path self-test: a bounded wait that nothing satisfies; after
+    ~2 s of GPU time err[0] holds CS_ERR_TIMEOUT."""
+    check(lib.cs_selftest_bounded_wait(_ptr(err), _stream(stream)))

@@ -8,6 +8,7 @@
 #include <cuda.h>
 
 #include "common.cuh"
+#include "ptx.cuh"
 #include "tma_host.h"
 
 namespace cs {
@@ -93,7 +94,29 @@ cs_status make_tmap(CUtensorMap* map, const void* base, int rank, const uint64_t
   return CS_OK;
 }
 
+// One thread waits on an mbarrier that nothing arrives on: the bounded wait that every
+// kernel of this library uses gives up after CS_WAIT_TIMEOUT_NS and records the timeout
+// in the device error word, and the kernel returns normally.
+__global__ void bounded_wait_selftest_kernel(int* err) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  block_sync();
+  if (threadIdx.x == 0) mbar_wait(&bar, 0, &abort_flag, err);   // phase 0 never completes
+}
+
 }  // namespace cs
+
+extern "C" cs_status cs_selftest_bounded_wait(int* err_dev, cudaStream_t stream) {
+  CS_REQUIRE(err_dev, "cs_selftest_bounded_wait: null error word");
+  cs::bounded_wait_selftest_kernel<<<1, 32, 0, stream>>>(err_dev);
+  CS_LAUNCHED();
+  return CS_OK;
+}
 
 extern "C" const char* cs_last_error(void) { return cs::g_last_error.c_str(); }
 extern "C" const char* cs_version(void) { return "cachedsearch-gb300 0.1 (sm_103a)"; }

@@ -67,3 +67,8 @@ def test_streamed_generator_matches_flat_layout(b):
     assert [i for i, _ in parts] == list(range(len(parts)))
     assert len(parts) == b.lib.cs_param_tensor_count(C.byref(b.model_config(m, 1)))
     assert np.array_equal(np.concatenate([a.reshape(-1) for _, a in parts]), flat)
+
+
+def test_failure_selftest_rejects_a_null_error_word_on_the_host(b):
+    st = b.lib.cs_selftest_bounded_wait(None, None)   # checked before any launch
+    assert st == b.CS_ERR_ARG and "null" in b.last_error()
