@@ -62,11 +62,11 @@ struct AttnCfg {
   static constexpr uint32_t IDESC_O = idesc_bf16_f32(128, HD);
 };
 
-template <int HD>
-__global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
-    attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                        const __grid_constant__ CUtensorMap tmV, const AttnArgs p) {
+template <int HD, bool TMA_O>
+__device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensorMap& tmK, const CUtensorMap& tmV,
+                                          const CUtensorMap& tmO, const AttnArgs& p) {
   using Cfg = AttnCfg<HD>;
+  static_assert(!TMA_O || HD % 64 == 0, "TMA output boxes are 64 columns wide");
   constexpr int NS = Cfg::NSTAGE;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -81,7 +81,8 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
   uint64_t* o_done = p_full + 2;           // [2]
   uint64_t* tok = o_done + 2;              // [2]: tok[g] = tile g may start its next MMA group
   uint64_t* teardown = tok + 2;            // [2]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(teardown + 2);
+  uint64_t* o_staged = teardown + 2;       // [2] (TMA_O): tile g's normalised O is in shared memory
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_staged + (TMA_O ? 2 : 0));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -105,6 +106,7 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
     for (int g = 0; g < 2; ++g) {
       mbar_init(&tok[g], 1);
       mbar_init(&teardown[g], 1);
+      if (TMA_O) mbar_init(&o_staged[g], 128);
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -298,7 +300,42 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
     }
     // final: O / l -> bf16
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&o_done[g], (nt - 1) & 1, abort_flag, p.err));
-    if (ok) {
+    if constexpr (TMA_O) {
+      // Rows go through the tile's own Q buffer (every MMA that read it has completed: the
+      // last o_done commit covers them) in the 128-byte-swizzled layout of a TMA box of
+      // 64 columns x 128 rows; one thread of the tile then stores the boxes (rows past Lq
+      // are clipped by the tensor map).
+      uint8_t* stg = sQ + g * Cfg::Q_BYTES;
+      if (ok) {
+        tc_fence_after();
+        const float inv_l = 1.f / l_run;
+#pragma unroll 1
+        for (int c = 0; c < HD / 32; ++c) {
+          uint32_t u[32];
+          tmem_ld32(tO + c * 32, u);
+          uint8_t* rowp = stg + (c >> 1) * Cfg::CH_BYTES + r * 128;
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+            uint4 o4;
+            o4.x = pack_bf16x2(__uint_as_float(u[8 * w + 0]) * inv_l, __uint_as_float(u[8 * w + 1]) * inv_l);
+            o4.y = pack_bf16x2(__uint_as_float(u[8 * w + 2]) * inv_l, __uint_as_float(u[8 * w + 3]) * inv_l);
+            o4.z = pack_bf16x2(__uint_as_float(u[8 * w + 4]) * inv_l, __uint_as_float(u[8 * w + 5]) * inv_l);
+            o4.w = pack_bf16x2(__uint_as_float(u[8 * w + 6]) * inv_l, __uint_as_float(u[8 * w + 7]) * inv_l);
+            const int unit = (c & 1) * 4 + w;
+            *reinterpret_cast<uint4*>(rowp + ((unit ^ (r & 7)) << 4)) = o4;
+          }
+        }
+        fence_proxy_async_smem();
+        mbar_arrive(&o_staged[g]);
+        if (qtr == 0 && lane == 0 && q0 + g * 128 < p.Lq && mbar_wait(&o_staged[g], 0, abort_flag, p.err)) {
+#pragma unroll
+          for (int c2 = 0; c2 < HD / 64; ++c2)
+            tma_store_3d(&tmO, stg + c2 * Cfg::CH_BYTES, head * HD + c2 * 64, q0 + g * 128, jb);
+          bulk_commit();
+          bulk_wait_all();   // the writes are done before the CTA's shared memory goes away
+        }
+      }
+    } else if (ok) {
       tc_fence_after();
       const int q = q0 + g * 128 + r;
       const float inv_l = 1.f / l_run;
@@ -331,13 +368,28 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
   }
 }
 
+// Two entry points so that the kernel with per-thread O stores keeps its three tensor maps.
+template <int HD>
+__global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
+    attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                        const __grid_constant__ CUtensorMap tmV, const AttnArgs p) {
+  attn_body<HD, false>(tmQ, tmK, tmV, tmQ, p);
+}
+template <int HD>
+__global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
+    attn_tcgen05_tma_o_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                              const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
+                              const AttnArgs p) {
+  attn_body<HD, true>(tmQ, tmK, tmV, tmO, p);
+}
+
 template <int HD>
 static cs_status launch_attn(const void* q, const void* k, const void* vt, void* o, int B, int heads, int Lq, int Lk,
                              int Lkv_stride, int kv_shared, int kv_sets, const int32_t* item_idx, int x_rows,
                              int* err, cudaStream_t stream) {
   using Cfg = AttnCfg<HD>;
   const int BH = B * heads, Bkv = kv_shared ? heads * kv_sets : BH;
-  CUtensorMap tq, tk, tv;
+  CUtensorMap tq, tk, tv, to;
   {
     const uint64_t dims[3] = {(uint64_t)Cfg::HDS, (uint64_t)Lq, (uint64_t)BH};
     const uint64_t str[2] = {(uint64_t)Cfg::HDS * 2, (uint64_t)Lq * Cfg::HDS * 2};
@@ -356,15 +408,36 @@ static cs_status launch_attn(const void* q, const void* k, const void* vt, void*
     const uint32_t box[3] = {64, (uint32_t)HD, 1};
     CS_TRY(make_tmap_bf16(&tv, vt, 3, dims, str, box));
   }
+  // O through TMA stores pays off when the key loop is short (cross-attention: the epilogue
+  // is a third of a CTA); with long key loops it measured slower (the kernel's registers
+  // are tight), so there each thread stores its own rows.
+  const bool tma_o = HD % 64 == 0 && Lk <= 2048;
+  to = tq;   // unused unless tma_o
+  if (tma_o) {
+    // O [B][Lq][heads*hd]: 64-column x 128-row boxes, clipped at Lq within each batch item
+    const uint64_t dims[3] = {(uint64_t)heads * HD, (uint64_t)Lq, (uint64_t)B};
+    const uint64_t str[2] = {(uint64_t)heads * HD * 2, (uint64_t)Lq * heads * HD * 2};
+    const uint32_t box[3] = {64, 128, 1};
+    CS_TRY(make_tmap_bf16(&to, o, 3, dims, str, box));
+  }
   AttnArgs a{};
   a.B = B; a.heads = heads; a.Lq = Lq; a.Lk = Lk; a.kv_shared = kv_shared;
   a.item_idx = item_idx; a.x_rows = x_rows > 0 ? x_rows : 1;
   a.scale_log2 = 1.4426950408889634f / sqrtf((float)HD);
   a.o = static_cast<__nv_bfloat16*>(o);
   a.err = err;
+  dim3 grid((Lq + 255) / 256, BH);
+  if constexpr (HD % 64 == 0) {
+    if (tma_o) {
+      auto kern = attn_tcgen05_tma_o_kernel<HD>;
+      CS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
+      kern<<<grid, Cfg::THREADS, Cfg::SMEM, stream>>>(tq, tk, tv, to, a);
+      CS_LAUNCHED();
+      return CS_OK;
+    }
+  }
   auto kern = attn_tcgen05_kernel<HD>;
   CS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
-  dim3 grid((Lq + 255) / 256, BH);
   kern<<<grid, Cfg::THREADS, Cfg::SMEM, stream>>>(tq, tk, tv, a);
   CS_LAUNCHED();
   return CS_OK;
