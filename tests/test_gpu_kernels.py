@@ -148,6 +148,7 @@ def _attn_case(B, hd, heads, nb, Lq, Lk, kv_shared, qscale, seed, kramp=0.0):
     (32, 4, 2, 48, 16, True, 2.0),         # tiny cross-attention, 16 text tokens
     (128, 2, 1, 1, 129, False, 1.0),       # one query row; the last key tile holds one key
     (128, 2, 2, 256, 1, False, 1.0),       # a single key: one tile, one valid column
+    (128, 1, 2, 300, 2100, False, 1.0),    # more than 2048 keys: per-thread output stores, ragged rows
 ])
 def test_attention_matches_oracle(B, hd, heads, nb, Lq, Lk, kv_shared, qscale):
     q, k, v, got = _attn_case(B, hd, heads, nb, Lq, Lk, kv_shared, qscale, seed=hd + Lq + Lk)
