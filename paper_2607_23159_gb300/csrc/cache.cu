@@ -136,6 +136,21 @@ __device__ __forceinline__ double warp_sum_partials(const float* __restrict__ p,
   return s;
 }
 
+// The drift's sums in the same order, in fp32: fp64 arithmetic on GB300 runs at a small
+// fraction of the fp32 rate, and its latency (~5 us per decision, measured) sat on the
+// critical path of the fused step.  256 chunk partials summed in fp32 add a relative
+// error of order 1e-6, far inside the 1e-3 near-tie zone of the decision.
+__device__ __forceinline__ float warp_sum_partials_f32(const float* __restrict__ p, int nch, int stride, int lane) {
+  float s = 0.f;
+  for (int c = lane; c < nch; c += 32) s += p[(long long)c * stride];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  return s;
+}
+
+// Relative drift of Eq. indicator from the two sums.
+__device__ __forceinline__ float drift_of(float num, float den) { return sqrtf(num) / sqrtf(den); }
+
 // One warp per candidate: drift from the partials, accumulate, decide; then thread 0
 // writes the ordered compaction list.
 __global__ void decide_finalize_kernel(const float* __restrict__ partials, int nch, float* __restrict__ accum,
@@ -147,10 +162,10 @@ __global__ void decide_finalize_kernel(const float* __restrict__ partials, int n
   for (int i = warp; i < N; i += nw) {
     const bool had = has_ref[i] != 0;
     const bool free_step = !window_forced_step && had;
-    double num = 0.0, den = 0.0;
+    float num = 0.f, den = 0.f;
     if (free_step) {
-      num = warp_sum_partials(partials + (long long)i * nch * 2 + 0, nch, 2, lane);
-      den = warp_sum_partials(partials + (long long)i * nch * 2 + 1, nch, 2, lane);
+      num = warp_sum_partials_f32(partials + (long long)i * nch * 2 + 0, nch, 2, lane);
+      den = warp_sum_partials_f32(partials + (long long)i * nch * 2 + 1, nch, 2, lane);
     }
     if (lane == 0) {
       bool compute;
@@ -158,12 +173,12 @@ __global__ void decide_finalize_kernel(const float* __restrict__ partials, int n
       if (!free_step) {
         compute = true;
       } else {
-        const double drift = sqrt(num) / sqrt(den);
+        const float drift = drift_of(num, den);
         if (!isfinite(drift)) {
           record_error(err, CS_ERR_NONFINITE);
           compute = true;
         } else {
-          a = (float)((double)a + drift);
+          a = a + drift;
           compute = (tau <= 0.f) || (a > tau);
         }
       }
@@ -450,20 +465,20 @@ __global__ void __launch_bounds__(kCacheThreads) decide_skip_kernel(
   for (int i = c_lo + warp; i < c_hi; i += nw) {
     const bool hr = had[i] != 0;
     const bool free_step = !wf && hr;
-    double num = 0.0, den = 0.0;
+    float num = 0.f, den = 0.f;
     if (free_step) {
-      num = warp_sum_partials(partials + (long long)i * nch * 2 + 0, nch, 2, lane);
-      den = warp_sum_partials(partials + (long long)i * nch * 2 + 1, nch, 2, lane);
+      num = warp_sum_partials_f32(partials + (long long)i * nch * 2 + 0, nch, 2, lane);
+      den = warp_sum_partials_f32(partials + (long long)i * nch * 2 + 1, nch, 2, lane);
     }
     if (lane == 0) {
       bool compute = true;
       float a = a_s[i];
       if (free_step) {
-        const double drift = sqrt(num) / sqrt(den);
+        const float drift = drift_of(num, den);
         if (!isfinite(drift)) {
           if (blockIdx.x == 0) record_error(err, CS_ERR_NONFINITE);
         } else {
-          a = (float)((double)a + drift);
+          a = a + drift;
           compute = (tau <= 0.f) || (a > tau);
         }
       }
@@ -502,8 +517,8 @@ __global__ void __launch_bounds__(kCacheThreads) decide_skip_kernel(
     const float* yi = kScore ? target + lo : nullptr;
     const int n8 = (int)((hi - lo) >> 3);
     float acc[1] = {0.f};
-#pragma unroll 2
-    for (int e = threadIdx.x; e < n8; e += kCacheThreads) {
+#pragma unroll 4
+    for (int e = threadIdx.x; e < n8; e += kCacheThreads) {   // a chunk's four rounds of loads all in flight
       const F8 xv = ld8_once(xi + 8 * e), dv = ld8_once(di + 8 * e);
       float xn[8], vu[8];
 #pragma unroll
@@ -745,7 +760,9 @@ extern "C" cs_status cs_cache_decide_skip(float* x, const float* x_ref, const fl
     set_error("cs_cache_decide_skip: kernel does not fit on an SM");
     return CS_ERR_CUDA;
   }
-  int grid = num_sms() * (per_sm < 8 ? per_sm : 8);
+  // at most 4 CTAs per SM: a smaller cooperative grid launches and crosses the barrier
+  // faster, and 4 x 256 threads still keep enough loads in flight (measured on GB300)
+  int grid = num_sms() * (per_sm < 4 ? per_sm : 4);
   const int items = N * nch;
   if (grid > items) grid = items;
   void* args[] = {&x, (void*)&x_ref, (void*)&delta, &accum, &has_ref, &N, &D, (void*)&nch, &wf, &tau,

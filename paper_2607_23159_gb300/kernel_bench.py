@@ -5,7 +5,9 @@
   python -m paper_2607_23159_gb300.kernel_bench cache --N 16 --D 2096640
 
 Inputs are random device tensors (the timing does not depend on their values).  Prints
-one JSON line with the average launch time and the achieved TFLOP/s or GB/s.
+one JSON line with the average launch time and the achieved TFLOP/s or GB/s.  The cache
+step is timed launch by launch after an L2-evicting write (median), since back-to-back
+launches of it measure the host's launch rate rather than the kernel.
 
 ``--torch`` times PyTorch's own kernels on the same shape instead (informal comparators,
 never part of the library's path): ``scaled_dot_product_attention`` for attention,
@@ -29,6 +31,26 @@ def _time(fn, reps, warmup):
     e1.record()
     torch.cuda.synchronize()
     return e0.elapsed_time(e1) / reps
+
+
+def _time_cold(fn, reps, warmup):
+    """Median of single launches, each after a 256 MB write that evicts the L2 (the
+    way the cache step runs inside a search step, between DiT evaluations)."""
+    import torch
+    for _ in range(warmup):
+        fn()
+    flush = torch.empty(64 << 20, device="cuda")
+    times = []
+    for _ in range(reps):
+        flush.add_(1.0)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        fn()
+        e1.record()
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    times.sort()
+    return times[len(times) // 2]
 
 
 def main():
@@ -83,7 +105,7 @@ def main():
             d = torch.linalg.vector_norm(x - xr, dim=1) / torch.linalg.vector_norm(xr, dim=1)
             x.add_(x + delta, alpha=h)
             return d
-        ms = _time(run, a.reps, a.warmup)
+        ms = _time_cold(run, a.reps, a.warmup)
         out.update(shape=dict(N=N, D=D, skipped=N), ms=ms, gbs=16.0 * N * D / (ms / 1e3) / 1e9)
     elif a.kernel == "attention":
         Lk = a.Lk or a.L
@@ -154,7 +176,7 @@ def main():
                 B.cache_decide(st["x"], st["x_ref"], st["accum"], st["has_ref"], 20, 50, 0.1, 5, 5, skip, idx, nc,
                                ws, force=force)
                 B.cache_apply(st["x"], st["x_ref"], st["delta"], v, skip, 0.6, 0.58)
-        ms = _time(run, a.reps, a.warmup)
+        ms = _time_cold(run, a.reps, a.warmup)
         n_skip = int((force == 0).sum())
         byts = (n_skip * 16.0 + (N - n_skip) * 24.0) * D
         out.update(shape=dict(N=N, D=D, skipped=n_skip), ms=ms, gbs=byts / (ms / 1e3) / 1e9)
