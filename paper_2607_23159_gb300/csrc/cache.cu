@@ -546,6 +546,21 @@ __global__ void __launch_bounds__(kCacheThreads) decide_skip_kernel(
   }
 }
 
+// A step inside the warm-up or cool-down window without a forced mask: every candidate
+// computes and no drift is evaluated (Sec. 3.1), so the decision needs no pass over the
+// latents and no grid-wide launch.
+__global__ void decide_all_compute_kernel(float* __restrict__ accum, uint8_t* __restrict__ has_ref, int N,
+                                          uint8_t* __restrict__ skip_mask, int32_t* __restrict__ idx,
+                                          int32_t* __restrict__ n_compute) {
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    accum[i] = 0.f;
+    has_ref[i] = 1;
+    skip_mask[i] = 0;
+    idx[i] = i;
+  }
+  if (threadIdx.x == 0) *n_compute = N;
+}
+
 // The update of computed candidates only (skipped ones were updated by decide_skip).
 template <bool kScore>
 __global__ void __launch_bounds__(kCacheThreads) apply_computed_kernel(
@@ -746,6 +761,11 @@ extern "C" cs_status cs_cache_decide_skip(float* x, const float* x_ref, const fl
              "cs_cache_decide_skip: needs D %% 8 == 0 and 32-byte aligned tensors");
   const int nch = cache_chunks(D);
   int wf = window_forced(step_k, T, K_w, K_c) ? 1 : 0;
+  if (wf && !force) {
+    decide_all_compute_kernel<<<1, 256, 0, stream>>>(accum, has_ref, N, skip_mask, idx, n_compute);
+    CS_LAUNCHED();
+    return CS_OK;
+  }
   float* partials = static_cast<float*>(workspace);
   float* spart = partials + (size_t)N * nch * 2;
   unsigned* bar = reinterpret_cast<unsigned*>(static_cast<char*>(workspace) + barrier_offset(N, D));
