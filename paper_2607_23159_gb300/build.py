@@ -5,6 +5,7 @@ library with no dependency on torch.  Run ``python -m paper_2607_23159_gb300.bui
 """
 from __future__ import annotations
 
+import fcntl
 import os
 import shutil
 import subprocess
@@ -44,9 +45,20 @@ def _compile(src: str, extra) -> str:
 
 
 def build(verbose_ptxas: bool = False, force: bool = False) -> str:
-    """Compile every kernel source and link the library; returns its path."""
+    """Compile every kernel source and link the library; returns its path.  Processes
+    that build at the same time (one per GPU rank) take turns on a lock file, so the
+    later ones find the library up to date."""
     os.makedirs(BUILD, exist_ok=True)
     os.makedirs(LIB_DIR, exist_ok=True)
+    with open(os.path.join(BUILD, ".lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)
+        try:
+            return _build_locked(verbose_ptxas, force)
+        finally:
+            fcntl.flock(lock, fcntl.LOCK_UN)
+
+
+def _build_locked(verbose_ptxas: bool, force: bool) -> str:
     srcs = sources()
     headers = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".cuh", ".h"))]
     headers += [os.path.join(ROOT, "include", f) for f in os.listdir(os.path.join(ROOT, "include"))]
