@@ -36,7 +36,10 @@ typedef enum {
   CS_ERR_NONFINITE = 3,   /* a norm in the drift indicator was NaN/Inf or ||x_ref|| = 0   */
   CS_ERR_TIMEOUT = 4,     /* a bounded device-side wait ran out                          */
   CS_ERR_NOMEM = 5,       /* device allocation failed                                    */
-  CS_ERR_UNSUPPORTED = 6  /* shape outside what the kernels implement                    */
+  CS_ERR_UNSUPPORTED = 6, /* shape outside what the kernels implement                    */
+  CS_ERR_BOUNDS = 7       /* index-checking build only (cs_build_flags() bit 0): a device
+                             index read from memory was out of range; the access was
+                             skipped and the error recorded in the device error word    */
 } cs_status;
 
 /* Shape of the DiT velocity model v_theta(x, t, c) (Sec. 2) and of its latent. */
@@ -59,6 +62,14 @@ const char* cs_last_error(void);
 
 /* Library version string. */
 const char* cs_version(void);
+
+/* Build options: bit 0 set when the library was compiled with CS_DEBUG_CHECKS (built by
+ * `python -m paper_2607_23159_gb300.build --debug` as lib/libcachedsearch_debug.so).
+ * That build checks every index the kernels read from device memory (the compaction list
+ * of computing candidates, the guidance K/V set of an item) before using it, records
+ * CS_ERR_BOUNDS in the device error word on a violation and skips the access; results are
+ * otherwise bit-identical to the normal build.  It stands in for a device memory checker. */
+int cs_build_flags(void);
 
 /* Number of float32 parameters of a model of this shape (the length of the flat
  * buffer cs_load_weights takes).  Layout, in order, Linear weights stored [out][in]

@@ -13,14 +13,18 @@ import os
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_HERE, "lib", "libcachedsearch.so")
+# CS_LIBRARY_VARIANT=debug selects the build with device-side index checks
+# (`python -m paper_2607_23159_gb300.build --debug`); anything else the normal build
+_VARIANT = os.environ.get("CS_LIBRARY_VARIANT", "release")
+LIB_PATH = os.path.join(_HERE, "lib", "libcachedsearch_debug.so" if _VARIANT == "debug" else "libcachedsearch.so")
 
 if not os.path.exists(LIB_PATH):
-    raise ImportError(f"{LIB_PATH} is missing: build it with `python -m paper_2607_23159_gb300.build` "
-                      "(or __graft_entry__.build())")
+    raise ImportError(f"{LIB_PATH} is missing: build it with `python -m paper_2607_23159_gb300.build"
+                      f"{' --debug' if _VARIANT == 'debug' else ''}` (or __graft_entry__.build())")
 lib = C.CDLL(LIB_PATH)
 
-CS_OK, CS_ERR_ARG, CS_ERR_CUDA, CS_ERR_NONFINITE, CS_ERR_TIMEOUT, CS_ERR_NOMEM, CS_ERR_UNSUPPORTED = range(7)
+(CS_OK, CS_ERR_ARG, CS_ERR_CUDA, CS_ERR_NONFINITE, CS_ERR_TIMEOUT, CS_ERR_NOMEM, CS_ERR_UNSUPPORTED,
+ CS_ERR_BOUNDS) = range(8)
 EPI_F32, EPI_BF16, EPI_GELU_BF16, EPI_RESID_F32, EPI_QKV = range(5)
 KC_SELF_ATTN, KC_CROSS_ATTN, KC_GEMM, KC_CACHE, KC_OTHER = range(5)
 
@@ -42,6 +46,7 @@ _SIGS = {
     "cs_selftest_bounded_wait": (I, [P, P]),
     "cs_last_error": (C.c_char_p, []),
     "cs_version": (C.c_char_p, []),
+    "cs_build_flags": (I, []),
     "cs_param_count": (SZ, [C.POINTER(ModelConfig)]),
     "cs_init_model": (I, [C.POINTER(ModelConfig), C.POINTER(P)]),
     "cs_destroy_model": (I, [P]),
@@ -94,6 +99,11 @@ def check(status: int):
 
 def launch_count() -> int:
     return int(lib.cs_launch_count())
+
+
+def index_checks() -> bool:
+    """True when the loaded library is the build with device-side index checks."""
+    return bool(lib.cs_build_flags() & 1)
 
 
 # ---------------------------------------------------------------- helpers --

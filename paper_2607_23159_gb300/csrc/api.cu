@@ -452,12 +452,15 @@ static cs_status dit_forward_impl(cs_model* m, const float* x, const int32_t* id
   if (n_c == 0) return CS_OK;
   const cs_model_config& c = m->cfg;
   const int d = c.d, L = m->L, M = n_c * L;
+  // valid state indices, checked by builds with CS_DEBUG_CHECKS: the search steps name
+  // states [0, x_rows * kv_sets); a caller of cs_dit_forward any non-negative row
+  const long long idx_limit = x_rows == (1 << 30) ? (1ll << 62) : (long long)x_rows * kv_sets;
   cudaEvent_t ev[2];
   CS_TRY(record_begin(m, 4, s, ev));
   cs::CondWeights cw{d, c.f_dim, c.blocks, m->time_w1, m->time_w2, m->mod_w, m->head_mod_w,
                      m->time_b1, m->time_b2, m->mod_b, m->head_mod_b, m->mod_offs_dev};
   CS_TRY(cs::timestep_conditioning(cw, t, m->cond_scratch, m->mods, m->hmod, s));
-  CS_TRY(cs::patchify(x, idx, n_c, x_rows, c.C, c.F, c.H, c.W, m->Kp, m->tok, s));
+  CS_TRY(cs::patchify(x, idx, n_c, x_rows, c.C, c.F, c.H, c.W, m->Kp, m->tok, idx_limit, m->err, s));
   CS_TRY(record_end(m, 4, s, ev, 0.0));
   CS_TRY(gemm(m, m->tok, m->patch_w, CS_EPI_F32, m->patch_b, nullptr, m->resid, d, M, d, m->Kp, s));
   const size_t kt = (size_t)c.heads * c.Lt * m->hd_s, vtt = (size_t)c.heads * m->hd * m->Ltv;
@@ -492,7 +495,7 @@ static cs_status dit_forward_impl(cs_model* m, const float* x, const int32_t* id
   CS_TRY(record_end(m, 4, s, ev, 0.0));
   CS_TRY(gemm(m, m->hbuf, m->head_w, CS_EPI_F32, m->head_b, nullptr, m->hout, m->P, M, m->P, d, s));
   CS_TRY(record_begin(m, 4, s, ev));
-  CS_TRY(cs::unpatchify(m->hout, idx, n_c, c.C, c.F, c.H, c.W, v, s));
+  CS_TRY(cs::unpatchify(m->hout, idx, n_c, c.C, c.F, c.H, c.W, v, idx_limit, m->err, s));
   CS_TRY(record_end(m, 4, s, ev, 0.0));
   return CS_OK;
 }

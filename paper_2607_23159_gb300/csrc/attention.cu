@@ -36,7 +36,7 @@ namespace cs {
 struct AttnArgs {
   int B, heads, Lq, Lk, kv_shared;
   const int32_t* item_idx;   // optional: shared K/V set of batch item j is item_idx[j] / x_rows
-  int x_rows;
+  int x_rows, kv_sets;
   float scale_log2;
   __nv_bfloat16* o;
   int* err;
@@ -88,7 +88,9 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensor
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int bh = blockIdx.y;
   const int head = bh % p.heads, jb = bh / p.heads;
-  const int bkv = !p.kv_shared ? bh : (p.item_idx ? (p.item_idx[jb] / p.x_rows) * p.heads + head : head);
+  int kv_set = p.kv_shared && p.item_idx ? p.item_idx[jb] / p.x_rows : 0;
+  if (!index_ok(kv_set, p.kv_sets, p.err)) kv_set = 0;
+  const int bkv = !p.kv_shared ? bh : kv_set * p.heads + head;
   const int q0 = blockIdx.x * 256;
   const int nt = (p.Lk + Cfg::BKV - 1) / Cfg::BKV;
 
@@ -422,7 +424,7 @@ static cs_status launch_attn(const void* q, const void* k, const void* vt, void*
   }
   AttnArgs a{};
   a.B = B; a.heads = heads; a.Lq = Lq; a.Lk = Lk; a.kv_shared = kv_shared;
-  a.item_idx = item_idx; a.x_rows = x_rows > 0 ? x_rows : 1;
+  a.item_idx = item_idx; a.x_rows = x_rows > 0 ? x_rows : 1; a.kv_sets = kv_sets;
   a.scale_log2 = 1.4426950408889634f / sqrtf((float)HD);
   a.o = static_cast<__nv_bfloat16*>(o);
   a.err = err;

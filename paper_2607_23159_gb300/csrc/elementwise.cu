@@ -70,7 +70,8 @@ cs_status layernorm_modulate(const float* x, const float* shift, const float* sc
 // tokens[j*L + l][k]: for k < 4C, element (c, f, 2hh+ph, 2ww+pw) of candidate idx[j]
 // with k = 4c + 2ph + pw and l = (f*(H/2) + hh)*(W/2) + ww; columns 4C..Kp-1 are 0.
 __global__ void patchify_kernel(const float* __restrict__ x, const int32_t* __restrict__ idx, int n_c, int x_rows,
-                                int C, int F, int H, int W, int Kp, __nv_bfloat16* __restrict__ tok) {
+                                int C, int F, int H, int W, int Kp, __nv_bfloat16* __restrict__ tok,
+                                long long idx_limit, int* err) {
   const int L = F * (H / 2) * (W / 2);
   const long long total = (long long)n_c * L * Kp;
   const long long D = (long long)C * F * H * W;
@@ -80,7 +81,7 @@ __global__ void patchify_kernel(const float* __restrict__ x, const int32_t* __re
     const long long row = t / Kp;
     const int l = (int)(row % L), j = (int)(row / L);
     float v = 0.f;
-    if (k < 4 * C) {
+    if (k < 4 * C && index_ok(idx[j], idx_limit, err)) {
       const int c = k >> 2, ph = (k >> 1) & 1, pw = k & 1;
       const int ww = l % (W / 2), hh = (l / (W / 2)) % (H / 2), f = l / ((W / 2) * (H / 2));
       v = x[(long long)(idx[j] % x_rows) * D + (((long long)c * F + f) * H + (2 * hh + ph)) * W + (2 * ww + pw)];
@@ -91,7 +92,7 @@ __global__ void patchify_kernel(const float* __restrict__ x, const int32_t* __re
 
 // v[idx[j]][c][f][h][w] = hout[(j*L + l)*P + 4c + 2(h%2) + (w%2)]
 __global__ void unpatchify_kernel(const float* __restrict__ hout, const int32_t* __restrict__ idx, int n_c, int C,
-                                  int F, int H, int W, float* __restrict__ v) {
+                                  int F, int H, int W, float* __restrict__ v, long long idx_limit, int* err) {
   const int L = F * (H / 2) * (W / 2), P = 4 * C;
   const long long D = (long long)C * F * H * W;
   const long long total = (long long)n_c * D;
@@ -102,24 +103,25 @@ __global__ void unpatchify_kernel(const float* __restrict__ hout, const int32_t*
     const int w = (int)(e % W), h = (int)((e / W) % H), f = (int)((e / ((long long)W * H)) % F);
     const int c = (int)(e / ((long long)W * H * F));
     const int l = (f * (H / 2) + h / 2) * (W / 2) + w / 2;
-    v[(long long)idx[j] * D + e] = hout[((long long)j * L + l) * P + 4 * c + 2 * (h & 1) + (w & 1)];
+    if (index_ok(idx[j], idx_limit, err))
+      v[(long long)idx[j] * D + e] = hout[((long long)j * L + l) * P + 4 * c + 2 * (h & 1) + (w & 1)];
   }
 }
 
 cs_status patchify(const float* x, const int32_t* idx, int n_c, int x_rows, int C, int F, int H, int W, int Kp,
-                   __nv_bfloat16* tok, cudaStream_t s) {
+                   __nv_bfloat16* tok, long long idx_limit, int* err, cudaStream_t s) {
   const long long total = (long long)n_c * F * (H / 2) * (W / 2) * Kp;
   const int blocks = (int)((total + 255) / 256 < 65535 * 16 ? (total + 255) / 256 : 65535 * 16);
-  patchify_kernel<<<blocks, 256, 0, s>>>(x, idx, n_c, x_rows, C, F, H, W, Kp, tok);
+  patchify_kernel<<<blocks, 256, 0, s>>>(x, idx, n_c, x_rows, C, F, H, W, Kp, tok, idx_limit, err);
   CS_LAUNCHED();
   return CS_OK;
 }
 
 cs_status unpatchify(const float* hout, const int32_t* idx, int n_c, int C, int F, int H, int W, float* v,
-                     cudaStream_t s) {
+                     long long idx_limit, int* err, cudaStream_t s) {
   const long long total = (long long)n_c * C * F * H * W;
   const int blocks = (int)((total + 255) / 256 < 65535 * 16 ? (total + 255) / 256 : 65535 * 16);
-  unpatchify_kernel<<<blocks, 256, 0, s>>>(hout, idx, n_c, C, F, H, W, v);
+  unpatchify_kernel<<<blocks, 256, 0, s>>>(hout, idx, n_c, C, F, H, W, v, idx_limit, err);
   CS_LAUNCHED();
   return CS_OK;
 }

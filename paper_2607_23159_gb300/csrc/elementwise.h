@@ -22,15 +22,16 @@ cs_status timestep_conditioning(const CondWeights& w, float t, float* scratch, f
 cs_status layernorm_modulate(const float* x, const float* shift, const float* scale, __nv_bfloat16* out, int M, int d,
                              cudaStream_t s);
 // tokens of latent rows idx[j] % x_rows (x_rows: rows of x; a cache state index may
-// exceed it when several states share a latent, as the two guidance branches do)
+// exceed it when several states share a latent, as the two guidance branches do);
+// idx_limit: valid state indices are [0, idx_limit) (checked in CS_DEBUG_CHECKS builds)
 cs_status patchify(const float* x, const int32_t* idx, int n_c, int x_rows, int C, int F, int H, int W, int Kp,
-                   __nv_bfloat16* tok, cudaStream_t s);
+                   __nv_bfloat16* tok, long long idx_limit, int* err, cudaStream_t s);
 // self/cross attention; with kv_sets > 1 batch item j uses shared K/V set item_idx[j] / x_rows
 cs_status attention_run(const void* q, const void* k, const void* vt, void* o, int B, int heads, int Lq, int Lk,
                         int hd, int Lkv_stride, int kv_shared, int kv_sets, const int32_t* item_idx, int x_rows,
                         int* err, cudaStream_t stream);
 cs_status unpatchify(const float* hout, const int32_t* idx, int n_c, int C, int F, int H, int W, float* v,
-                     cudaStream_t s);
+                     long long idx_limit, int* err, cudaStream_t s);
 cs_status to_bf16_pad(const float* src, long long rows, int cols, int ld, __nv_bfloat16* dst, cudaStream_t s);
 
 }  // namespace cs

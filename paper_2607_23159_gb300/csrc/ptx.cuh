@@ -16,6 +16,13 @@
 namespace cs {
 
 constexpr int kErrTimeout = 4;   // == CS_ERR_TIMEOUT in include/cachedsearch.h
+constexpr int kErrBounds = 7;    // == CS_ERR_BOUNDS
+
+#ifdef CS_DEBUG_CHECKS
+constexpr bool kIndexChecks = true;
+#else
+constexpr bool kIndexChecks = false;
+#endif
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -38,6 +45,15 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
 
 __device__ __forceinline__ void record_error(int* err, int code) {
   if (err) atomicCAS(err, 0, code);
+}
+
+// Index read from device memory, checked in builds with CS_DEBUG_CHECKS: outside
+// [0, limit) it records CS_ERR_BOUNDS and returns false so that the caller skips the
+// access.  Without the flag this is `true` and compiles away.
+__device__ __forceinline__ bool index_ok(long long i, long long limit, int* err) {
+  if (!kIndexChecks || (i >= 0 && i < limit)) return true;
+  record_error(err, kErrBounds);
+  return false;
 }
 
 // ------------------------------------------------------------------ mbarrier --

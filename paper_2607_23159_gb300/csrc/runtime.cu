@@ -120,4 +120,12 @@ extern "C" cs_status cs_selftest_bounded_wait(int* err_dev, cudaStream_t stream)
 
 extern "C" const char* cs_last_error(void) { return cs::g_last_error.c_str(); }
 extern "C" const char* cs_version(void) { return "cachedsearch-gb300 0.1 (sm_103a)"; }
+
+extern "C" int cs_build_flags(void) {
+#ifdef CS_DEBUG_CHECKS
+  return 1;
+#else
+  return 0;
+#endif
+}
 extern "C" long long cs_launch_count(void) { return cs::g_launches.load(); }
