@@ -258,3 +258,26 @@ def test_streamed_weight_loading_equals_flat_loading(B):
     assert torch.equal(va, vb)
     a.close()
     b.close()
+
+
+def test_host_buffer_step_equals_device_step_tiny(B, tiny):
+    """cs_search_step_host (latents and mask in pinned host memory, the path the bench's
+    end-to-end number takes) gives the device-buffer step's latents and masks bit for bit."""
+    cfg, inp, _ = tiny
+    st_d, m_d, _, n_d = gpu_search(B, inp, cfg.N, cfg.T, cfg.tau, cfg.K_w, cfg.K_c, score=False)
+    model = B.Model(cfg.model, cfg.N)
+    model.load_weights(inp.flat)
+    model.set_text_context(dev(inp.ctx))
+    xh = torch.from_numpy(inp.x1.reshape(cfg.N, -1).copy()).pin_memory()
+    skip_h = torch.zeros(cfg.N, dtype=torch.uint8).pin_memory()
+    st = B.new_state(cfg.N, cfg.model.D)
+    t = O.time_grid(cfg.T)
+    masks, ncs = [], []
+    for k in range(1, cfg.T + 1):
+        ncs.append(model.search_step_host(xh, st, k, cfg.T, float(t[k - 1]), float(t[k]), cfg.tau, cfg.K_w, cfg.K_c,
+                                          skip_h))
+        masks.append(skip_h.numpy().astype(bool).copy())
+    assert model.device_error() == 0
+    model.close()
+    assert ncs == n_d and np.array_equal(np.array(masks), m_d)
+    assert torch.equal(xh, st_d["x"].cpu())
