@@ -281,3 +281,44 @@ def test_host_buffer_step_equals_device_step_tiny(B, tiny):
     model.close()
     assert ncs == n_d and np.array_equal(np.array(masks), m_d)
     assert torch.equal(xh, st_d["x"].cpu())
+
+
+def test_kernel_stats_count_the_algorithmic_work(B, tiny):
+    """The per-class counters behind the bench's roofline: with every candidate forced to
+    compute, the GEMM, self- and cross-attention work equal the closed-form FLOPs of the
+    DiT per candidate-step (QKV 6Ld^2 ... per block), the cache class counts its
+    algorithmic bytes, and every class records launches and time."""
+    cfg, inp, _ = tiny
+    m, N, T = cfg.model, cfg.N, cfg.T
+    model = B.Model(m, N)
+    model.load_weights(inp.flat)
+    model.set_text_context(dev(inp.ctx))
+    st = B.new_state(N, m.D)
+    st["x"].copy_(dev(inp.x1.reshape(N, -1)))
+    skip = torch.zeros(N, dtype=torch.uint8, device="cuda")
+    force = torch.ones(N, dtype=torch.uint8, device="cuda")
+    t = O.time_grid(T)
+    model.reset_kernel_stats()
+    model.set_profiling(True)
+    for k in range(1, T + 1):
+        assert model.search_step(st, k, T, float(t[k - 1]), float(t[k]), cfg.tau, cfg.K_w, cfg.K_c, skip,
+                                 force=force) == N
+    model.set_profiling(False)
+    stats = {c: model.kernel_stats(c) for c in range(5)}
+    assert model.device_error() == 0
+    model.close()
+    L, d, hd, H, Lt, ffn, nb = m.L, m.d, m.hd, m.heads, m.Lt, m.ffn, m.blocks
+    P = 4 * m.C
+    Kp = (P + 63) // 64 * 64          # the patch embedding runs on zero-padded 64-wide rows
+    cs = N * T                        # computed candidate-steps
+    gemm = 2.0 * L * (d * Kp + nb * (6 * d * d + 2 * d * ffn) + P * d)
+    assert stats[B.KC_GEMM][2] == cs * gemm
+    assert stats[B.KC_SELF_ATTN][2] == cs * nb * 4.0 * H * L * L * hd
+    assert stats[B.KC_CROSS_ATTN][2] == cs * nb * 4.0 * H * L * Lt * hd
+    assert stats[B.KC_SELF_ATTN][0] == T * nb and stats[B.KC_CROSS_ATTN][0] == T * nb
+    # cache bytes: computed candidates read x, v and write x, Delta, x_ref (20 D), plus the
+    # x_ref read of the drift on free steps (24 D)
+    free = sum(1 for k in range(1, T + 1) if not (k <= cfg.K_w or k > T - cfg.K_c))
+    assert stats[B.KC_CACHE][2] == float(m.D * N * (20 * (T - free) + 24 * free))
+    for c in range(5):
+        assert stats[c][0] > 0 and stats[c][1] > 0.0, c
