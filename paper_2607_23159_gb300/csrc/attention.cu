@@ -9,8 +9,9 @@
 //                so that the tensor core works on one tile while the other's softmax runs
 //   warps 2..5   softmax of tile A, warps 6..9 softmax of tile B: one thread per query
 //                row (the warp's TMEM lane quarter), all 128 keys of the tile in
-//                registers.  Online softmax in log2 units with lazy O rescaling (only
-//                when the running max grows by more than 8).  P is written back to TMEM
+//                registers; the row maximum comes with the reducing TMEM load
+//                (tcgen05.ld.red).  Online softmax in log2 units with lazy O rescaling
+//                (only when the running max grows by more than 8).  P is written back to TMEM
 //                as bf16 over the row's own S columns and fed to the PV MMA as the TMEM
 //                A operand.
 //
@@ -243,24 +244,27 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensor
       if (!__all_sync(0xffffffffu, mbar_wait(&s_full[g], j & 1, abort_flag, p.err))) { ok = false; break; }
       tc_fence_after();
       uint32_t u[128];
-      tmem_ld128(tS, u);
+      float rmax;
       const int valid = p.Lk - j * Cfg::BKV;
-      if (valid < Cfg::BKV) {
+      if (valid >= Cfg::BKV) {
+        tmem_ld128_max(tS, u, rmax);            // the row maximum comes with the load
+      } else {                                  // last, partial key tile: mask, then reduce
+        tmem_ld128(tS, u);
 #pragma unroll
         for (int e = 0; e < Cfg::BKV; ++e)
           if (e >= valid) u[e] = __float_as_uint(-INFINITY);
+        float mx[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) mx[q] = __uint_as_float(u[q]);
+#pragma unroll
+        for (int e = 4; e < Cfg::BKV - 4; e += 8) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q) mx[q] = fmax3(mx[q], __uint_as_float(u[e + 2 * q]), __uint_as_float(u[e + 2 * q + 1]));
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) mx[q] = fmaxf(mx[q], __uint_as_float(u[Cfg::BKV - 4 + q]));
+        rmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
       }
-      float mx[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) mx[q] = __uint_as_float(u[q]);
-#pragma unroll
-      for (int e = 4; e < Cfg::BKV - 4; e += 8) {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) mx[q] = fmax3(mx[q], __uint_as_float(u[e + 2 * q]), __uint_as_float(u[e + 2 * q + 1]));
-      }
-#pragma unroll
-      for (int q = 0; q < 4; ++q) mx[q] = fmaxf(mx[q], __uint_as_float(u[Cfg::BKV - 4 + q]));
-      const float rmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
       const float m_new = fmaxf(m_run, rmax * sl2);
       const bool need = (j == 0) || (m_new > m_run + 8.f);
       const bool warp_need = __any_sync(0xffffffffu, need);
