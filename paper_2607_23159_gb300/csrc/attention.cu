@@ -171,39 +171,49 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensor
       const uint32_t q_base = smem_u32(sQ);
       const uint32_t sdst = tmem_base + g * 128, odst = tmem_base + 256 + g * HD;
       const uint64_t ad = sdesc_sw128(q_base + g * Cfg::Q_BYTES);
-      // Descriptors are built once per tile; the k-th slice adds its byte offset / 16 to the
-      // start-address field (shared addresses stay below 2^18, so the field cannot carry).
-      auto issue_s = [&](uint32_t kslot, uint64_t* pass) {
-        const uint64_t bd = sdesc_sw128(kslot);
+      // Every descriptor of both ring stages is built once (shared addresses stay below 2^18,
+      // so adding a slice's byte offset / 16 to the start-address field cannot carry); the
+      // MMAs go out four to an asm block, which keeps the issuing thread's instruction
+      // count per MMA low (its sub-partition is shared with softmax warps).
+      static_assert(Cfg::NSTAGE == 2 && Cfg::HANDOVER == 4, "descriptor tables: two stages, hand-over at 4");
+      constexpr int NKS = Cfg::HDS / 16;      // K slices of S (4 or 8)
+      auto v_addr = [&](int st) { return smem_u32(sKV + (st % NS) * 2 * Cfg::SLOT); };
+      auto k_addr = [&](int st) { return v_addr(st) + Cfg::SLOT; };
+      uint64_t qa[8], kb0[8], kb1[8], vb0[8], vb1[8];
+      uint32_t pa[8];
 #pragma unroll
-        for (int kk = 0; kk < Cfg::HDS / 16; ++kk) {
-          if (pass && kk == Cfg::HDS / 16 - Cfg::HANDOVER) mbar_arrive(pass);
-          const uint64_t off = (uint64_t)(((kk >> 2) * Cfg::CH_BYTES + (kk & 3) * 32) >> 4);
-          umma_bf16_ss(sdst, ad + off, bd + off, Cfg::IDESC_S, kk > 0 ? 1u : 0u);
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint64_t offk = (uint64_t)(((kk >> 2) * Cfg::CH_BYTES + (kk & 3) * 32) >> 4);
+        const uint64_t offv = (uint64_t)(((kk >> 2) * Cfg::VCH_BYTES + (kk & 3) * 32) >> 4);
+        qa[kk] = ad + offk;
+        kb0[kk] = sdesc_sw128(k_addr(0)) + offk;
+        kb1[kk] = sdesc_sw128(k_addr(1)) + offk;
+        vb0[kk] = sdesc_sw128(v_addr(0)) + offv;
+        vb1[kk] = sdesc_sw128(v_addr(1)) + offv;
+        pa[kk] = sdst + (kk >> 2) * 64 + (kk & 3) * 8;   // keys 16kk..: half kk/4, packed pairs
+      }
+      auto issue_s = [&](const uint64_t* kb, uint64_t* pass) {
+        if (pass && NKS == Cfg::HANDOVER) mbar_arrive(pass);
+        umma4_ss(sdst, qa, kb, Cfg::IDESC_S, 0u);
+        if (NKS == 8) {
+          if (pass) mbar_arrive(pass);
+          umma4_ss(sdst, qa + 4, kb + 4, Cfg::IDESC_S, 1u);
         }
         umma_commit(&s_full[g]);
       };
-      auto issue_pv = [&](uint32_t vslot, int j, uint64_t* pass) {
-        const uint64_t bd = sdesc_sw128(vslot);
-#pragma unroll
-        for (int kk = 0; kk < Cfg::BKV / 16; ++kk) {
-          if (pass && kk == Cfg::BKV / 16 - Cfg::HANDOVER) mbar_arrive(pass);
-          // keys 16kk..16kk+15: half kk/4, packed bf16 pairs at columns 8*(kk%4) of that half
-          const uint64_t offb = (uint64_t)(((kk >> 2) * Cfg::VCH_BYTES + (kk & 3) * 32) >> 4);
-          umma_bf16_ts(odst, sdst + (kk >> 2) * 64 + (kk & 3) * 8, bd + offb, Cfg::IDESC_O,
-                       (j > 0 || kk > 0) ? 1u : 0u);
-        }
+      auto issue_pv = [&](const uint64_t* vb, int j, uint64_t* pass) {
+        umma4_ts(odst, pa, vb, Cfg::IDESC_O, j > 0 ? 1u : 0u);
+        if (pass) mbar_arrive(pass);
+        umma4_ts(odst, pa + 4, vb + 4, Cfg::IDESC_O, 1u);
         umma_commit(&o_done[g]);   // measured: this commit after each PV group runs faster than none
       };
-      auto v_addr = [&](int st) { return smem_u32(sKV + (st % NS) * 2 * Cfg::SLOT); };
-      auto k_addr = [&](int st) { return v_addr(st) + Cfg::SLOT; };
       uint64_t* other = &tok[1 - g];
       bool ok = mbar_wait(q_full, 0, abort_flag, p.err);
       if (ok) ok = mbar_wait(&kv_full[0], 0, abort_flag, p.err);
       if (ok && g == 1) ok = mbar_wait(&tok[1], 0, abort_flag, p.err);    // after S_A(0)
       if (ok) {
         tc_fence_after();
-        issue_s(k_addr(0), other);
+        issue_s(kb0, other);
         umma_commit(&kv_empty[0]);
       }
       // Token phases: tok[1] completes for S_A(0), then once per group A(j); tok[0] for
@@ -219,8 +229,13 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensor
         tc_fence_after();
         // the group's last MMAs hand the token over (group B only when a group A follows)
         uint64_t* pass = (g == 0 || more) ? other : nullptr;
-        issue_pv(v_addr(st), j, more ? nullptr : pass);
-        if (more) issue_s(k_addr(st), pass);
+        if ((st % NS) == 0) {   // two copies of the group, so the tables stay in registers
+          issue_pv(vb0, j, more ? nullptr : pass);
+          if (more) issue_s(kb0, pass);
+        } else {
+          issue_pv(vb1, j, more ? nullptr : pass);
+          if (more) issue_s(kb1, pass);
+        }
         umma_commit(&kv_empty[st % NS]);
       }
       if (*abort_flag) {
