@@ -256,7 +256,7 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensor
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     for (int j = 0; j < nt; ++j) {
-      if (!__all_sync(0xffffffffu, mbar_wait(&s_full[g], j & 1, abort_flag, p.err))) { ok = false; break; }
+      if (!__all_sync(0xffffffffu, mbar_wait_suspend(&s_full[g], j & 1, abort_flag, p.err))) { ok = false; break; }
       tc_fence_after();
       uint32_t u[128];
       float rmax;
@@ -320,7 +320,7 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensor
       mbar_arrive(&p_full[g]);
     }
     // final: O / l -> bf16
-    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&o_done[g], (nt - 1) & 1, abort_flag, p.err));
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait_suspend(&o_done[g], (nt - 1) & 1, abort_flag, p.err));
     if constexpr (TMA_O) {
       // Rows go through the tile's own Q buffer (every MMA that read it has completed: the
       // last o_done commit covers them) in the 128-byte-swizzled layout of a TMA box of

@@ -102,6 +102,37 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   }
 }
 
+// The same bounded wait for warps that have nothing else to do meanwhile: each poll
+// suspends the thread for up to 20 us (it wakes when the phase completes), so waiting warps
+// leave their sub-partition's issue slots to the warps that work, such as an MMA issuer.
+__device__ __forceinline__ uint32_t mbar_try_wait_suspend(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(20000u)
+      : "memory");
+  return ok;
+}
+__device__ __forceinline__ bool mbar_wait_suspend(uint64_t* bar, uint32_t parity, volatile int* abort, int* err) {
+  const uint32_t a = smem_u32(bar);
+  if (mbar_try_wait_suspend(a, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+    #pragma unroll 1
+    for (int i = 0; i < 8; ++i)
+      if (mbar_try_wait_suspend(a, parity)) return true;
+    if (*abort) return false;
+    if (globaltimer_ns() - t0 > CS_WAIT_TIMEOUT_NS) {
+      *abort = 1;
+      record_error(err, kErrTimeout);
+      return false;
+    }
+  }
+}
+
 // Bounded wait used on teardown paths only (no abort check).
 __device__ __forceinline__ bool mbar_wait_teardown(uint64_t* bar, uint32_t parity) {
   const uint32_t a = smem_u32(bar);
