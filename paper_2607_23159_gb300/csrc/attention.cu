@@ -18,8 +18,12 @@
 // One softmax warp per tile on each SM sub-partition: a tcgen05.mma needs issue slots on
 // the issuer's sub-partition.  Measured on GB300, an N=128 MMA stream runs at 64 cycles per
 // MMA alone, ~72-76 next to one warp that issues every cycle (a mix of FMA, MUFU and
-// conversions, like the softmax) and ~90-110 next to two to four such warps; the layout with
-// two threads per row (18 warps) ran its MMAs at ~90-110 cycles, this one at ~85-92.
+// conversions, like the softmax) and ~90-110 next to two to four such warps; warps of only
+// MUFU or only conversions do not slow it, warps of FMA or ALU instructions do.  So the
+// softmax keeps its FMA/ALU count low (packed f32x2 arithmetic, the reducing load instead of
+// a max pass), its warps wait on barriers with suspending polls instead of spinning, and the
+// issuers precompute their descriptors and issue four MMAs per asm block.  The layout with
+// two threads per row (18 warps) ran its MMAs at ~90-110 cycles.
 //
 // TMEM (512 columns): S_A [0,128), S_B [128,256) (P_g, keys 64h..64h+63 packed in pairs,
 // aliases columns [64h, 64h+32) of S_g), O_A [256, 256+hd), O_B [256+hd, 256+2hd).  V is stored
