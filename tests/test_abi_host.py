@@ -74,3 +74,17 @@ def test_streamed_generator_matches_flat_layout(b):
 def test_failure_selftest_rejects_a_null_error_word_on_the_host(b):
     st = b.lib.cs_selftest_bounded_wait(None, None)   # checked before any launch
     assert st == b.CS_ERR_ARG and "null" in b.last_error()
+
+
+def test_index_checking_build_reports_its_flag():
+    """The --debug build variant compiles (cross-compiled here, no GPU needed), lands at its
+    own path and reports bit 0 of cs_build_flags; the default library does not."""
+    import subprocess
+    import sys
+    from paper_2607_23159_gb300 import build as bld
+    path = bld.build(debug=True)
+    assert path.endswith("libcachedsearch_debug.so") and os.path.exists(path)
+    code = ("import ctypes, sys; lib = ctypes.CDLL(sys.argv[1]); print(lib.cs_build_flags())")
+    out = subprocess.run([sys.executable, "-c", code, path], capture_output=True, text=True, timeout=120)
+    assert out.returncode == 0, out.stderr
+    assert out.stdout.strip() == "1"
