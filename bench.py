@@ -33,7 +33,7 @@ sys.path.insert(0, ROOT)
 METRIC = "candidate-denoising-steps/sec at Wan2.1-1.3B shape"
 # DRAM bytes (read + write) of one self-attention launch per (candidate, head) at 32760
 # tokens, hd 128, from the ncu capture in profiles/attn_tcgen05_hd128_L32760.md
-ATTN_DRAM_BYTES_PER_HEAD_L32760 = 394.0e6 / 12
+ATTN_DRAM_BYTES_PER_HEAD_L32760 = 384.8e6 / 12
 UNIT = "candidate-steps/s"
 
 

@@ -25,8 +25,8 @@
 // issuers precompute their descriptors and issue four MMAs per asm block.  The layout with
 // two threads per row (18 warps) ran its MMAs at ~90-110 cycles.
 //
-// TMEM (512 columns): S_A [0,128), S_B [128,256) (P_g, keys 64h..64h+63 packed in pairs,
-// aliases columns [64h, 64h+32) of S_g), O_A [256, 256+hd), O_B [256+hd, 256+2hd).  V is stored
+// TMEM (512 columns): S_A [0,128), S_B [128,256) (P_g, all 128 keys packed in pairs, aliases
+// columns [0, 64) of S_g: one 64-column store), O_A [256, 256+hd), O_B [256+hd, 256+2hd).  V is stored
 // transposed (V^T [hd][keys]) so that it is a K-major B operand in shared memory.
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -194,7 +194,7 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensor
         kb1[kk] = sdesc_sw128(k_addr(1)) + offk;
         vb0[kk] = sdesc_sw128(v_addr(0)) + offv;
         vb1[kk] = sdesc_sw128(v_addr(1)) + offv;
-        pa[kk] = sdst + (kk >> 2) * 64 + (kk & 3) * 8;   // keys 16kk..: half kk/4, packed pairs
+        pa[kk] = sdst + kk * 8;                          // keys 16kk..16kk+15 packed in 8 columns
       }
       auto issue_s = [&](const uint64_t* kb, uint64_t* pass) {
         if (pass && NKS == Cfg::HANDOVER) mbar_arrive(pass);
@@ -318,8 +318,7 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensor
           tmem_st32(tO + c * 32, o);
         }
       }
-      tmem_st32(tS, *reinterpret_cast<const uint32_t(*)[32]>(&u[0]));
-      tmem_st32(tS + 64, *reinterpret_cast<const uint32_t(*)[32]>(&u[32]));
+      tmem_st64(tS, u);                         // P: keys 2c, 2c+1 packed in column c
       tc_fence_before();
       mbar_arrive(&p_full[g]);
     }
