@@ -25,3 +25,24 @@ def test_reference_arm_prints_one_contract_line():
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+
+
+def test_clock_summary_parses_nvidia_smi_samples():
+    """The bench's `clocks` key: median SM clock under load, the maximum, and every
+    throttle reason seen active in any sample (what decides whether a run is kept)."""
+    sys.path.insert(0, ROOT)
+    import bench
+    clk = bench.ClockSampler(0)
+    clk.out = "\n".join([
+        "1920, 2070, 1100.5, Not Active, Not Active, Not Active, Active",
+        "1935, 2070, 1180.0, Not Active, Not Active, Not Active, Active",
+        "1890, 2070, 1200.2, Not Active, Active, Not Active, Not Active",
+        "garbage line",
+        "",
+    ])
+    s = clk.summary()
+    assert s["sm_mhz"] == 1920 and s["sm_max_mhz"] == 2070 and s["samples"] == 3
+    assert s["reasons"] == ["hw_thermal_slowdown", "sw_power_cap"]
+    empty = bench.ClockSampler(0)
+    empty.out = ""
+    assert empty.summary()["reasons"] == ["unsampled"]
