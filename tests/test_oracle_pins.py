@@ -127,10 +127,11 @@ def test_search_step_equals_per_candidate_rollout():
     xs = x1s.copy()
     masks = []
     for k in range(1, T + 1):
-        xs, skipped, _, _ = O.search_step(states, xs, k, T, 0.1, 1, 1, vel)
+        xs, skipped, _, _ = O.search_step(states, xs, k, T, 0.5, 1, 1, vel)
         masks.append(~skipped)
+    assert not np.array(masks).all()  # tau 0.5 skips steps 2 and 4: the states matter
     for i in range(3):
-        xf, comp, _ = O.rollout(x1s[i], T, 0.1, 1, 1, vel)
+        xf, comp, _ = O.rollout(x1s[i], T, 0.5, 1, 1, vel)
         assert np.array_equal(xf, xs[i])
         assert np.array_equal(comp, np.array(masks)[:, i])
 
@@ -145,8 +146,22 @@ def test_x0_estimate_score_on_last_step_is_final_latent_score():
     states = [O.CacheState() for _ in range(2)]
     xs = x1s
     for k in range(1, T + 1):
-        xs, _, _, sc = O.search_step(states, xs, k, T, 0.1, 1, 1, vel, target=y)
+        xs, _, _, sc = O.search_step(states, xs, k, T, 0.5, 1, 1, vel, target=y)
     np.testing.assert_allclose(sc, [-np.linalg.norm(xs[i] - y) for i in range(2)], rtol=1e-15)
+
+
+def test_x0_estimate_is_exact_for_a_constant_field():
+    # v = c: every trajectory is the straight line x_t = x_1 - (1 - t) c, so the x0
+    # estimate x_{k+1} - t_{k+1} v equals x_1 - c at every step, not only the last
+    c = np.array([0.4, -0.2, 1.5])
+    x1s = np.array([[1.0, 2.0, -1.0], [0.5, 0.0, 3.0]])
+    y = np.array([0.1, 0.2, 0.3])
+    T = 7
+    states = [O.CacheState() for _ in range(2)]
+    xs = x1s
+    for k in range(1, T + 1):
+        xs, _, _, sc = O.search_step(states, xs, k, T, 0.0, 0, 0, lambda x, t: c, target=y)
+        np.testing.assert_allclose(sc, [-np.linalg.norm(x1s[i] - c - y) for i in range(2)], rtol=1e-13)
 
 
 # --------------------------------------------------------- search / select ---
@@ -169,8 +184,9 @@ def test_cached_search_brute_force_argmax():
     x1s = synth.initial_noise(cfg, range(4))
     y = synth.target_latent(cfg)
     vel = lambda x, t: m.velocity(x, t, kv)
-    i_star, scores, finals, _ = O.cached_search(x1s, 5, 0.1, 1, 1, vel, y)
-    brute = [-np.sqrt(((O.rollout(x1s[i], 5, 0.1, 1, 1, vel)[0] - y) ** 2).sum()) for i in range(4)]
+    i_star, scores, finals, comp = O.cached_search(x1s, 5, 0.5, 1, 1, vel, y)
+    assert not comp.all()
+    brute = [-np.sqrt(((O.rollout(x1s[i], 5, 0.5, 1, 1, vel)[0] - y) ** 2).sum()) for i in range(4)]
     np.testing.assert_allclose(scores, brute, rtol=1e-15)
     assert scores[i_star] == max(scores)
 
@@ -299,6 +315,17 @@ def test_dit_token_permutation_equivariance():
     np.testing.assert_allclose(vp, v[perm], atol=1e-11)
 
 
+def test_dit_text_token_permutation_invariance():
+    # cross-attention sums over the text tokens: reordering them (keys and values
+    # together) leaves the velocity unchanged
+    cfg, m = _tiny_model()
+    ctx = synth.text_context(cfg)
+    perm = np.random.default_rng(6).permutation(cfg.Lt)
+    x = synth.initial_noise(cfg, [1])[0].astype(np.float64)
+    v = m.velocity(x, 0.4, m.text_kv(ctx))
+    np.testing.assert_allclose(m.velocity(x, 0.4, m.text_kv(np.asarray(ctx)[perm])), v, atol=1e-11)
+
+
 def test_dit_zero_blocks_reduce_to_head_of_embedding():
     # all block weights 0 (and biases 0): every block is the identity, so
     # v = head(LN(embed(x)) (1 + scale_h) + shift_h)
@@ -339,17 +366,18 @@ def test_beam_and_pruned_search_degenerate_cases():
     y = synth.target_latent(cfg)
     vel = lambda x, t: m.velocity(x, t, kv)
     T = 6
-    i_star, sc, _, _ = O.cached_search(x1s, T, 0.1, 1, 1, vel, y)
+    i_star, sc, _, _ = O.cached_search(x1s, T, 0.5, 1, 1, vel, y)
     # keep everything, no children: the beam only permutes slots
-    sb, _, _ = O.beam_search(x1s, T, 0.1, 1, 1, vel, y, every=2, keep=4, children=0, sigma=0.0,
+    sb, _, _ = O.beam_search(x1s, T, 0.5, 1, 1, vel, y, every=2, keep=4, children=0, sigma=0.0,
                              noise_for_round=lambda r: None)
     np.testing.assert_allclose(np.sort(sb), np.sort(sc), rtol=1e-12)
     # sigma = 0 children are exact copies of their parent
-    sb, xb, _ = O.beam_search(x1s, T, 0.1, 1, 1, vel, y, every=3, keep=2, children=1, sigma=0.0,
-                              noise_for_round=lambda r: np.ones((2, *x1s.shape[1:])))
+    sb, xb, skipped = O.beam_search(x1s, T, 0.5, 1, 1, vel, y, every=3, keep=2, children=1, sigma=0.0,
+                                    noise_for_round=lambda r: np.ones((2, *x1s.shape[1:])))
+    assert skipped[3:].any()  # children skip on the cache state they inherited
     assert np.array_equal(xb[0], xb[1]) and np.array_equal(xb[2], xb[3])
     # pruning that keeps every candidate picks the same winner as the plain search
-    win, sp, ids, _ = O.pruned_search(x1s, T, 0.1, 1, 1, vel, y, prune_step=3, keep=4)
+    win, sp, ids, _ = O.pruned_search(x1s, T, 0.5, 1, 1, vel, y, prune_step=3, keep=4)
     assert win == i_star
     np.testing.assert_allclose(np.sort(sp), np.sort(sc), rtol=1e-12)
 
