@@ -391,17 +391,6 @@ __device__ __forceinline__ void tmem_ld128_max(uint32_t taddr, uint32_t (&r)[128
       : "memory");
 }
 
-// D[tmem] (+)= A[tmem] * B[smem]^T (A: 128 lanes = rows, K packed two bf16 per column).
-__device__ __forceinline__ void umma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
-                                             uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-
 // Packed float32 pairs (sm_100+): d = a * b + c and d = a + b, element-wise on two lanes.
 __device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
   uint64_t r;
