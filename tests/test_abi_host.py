@@ -88,3 +88,26 @@ def test_index_checking_build_reports_its_flag():
     out = subprocess.run([sys.executable, "-c", code, path], capture_output=True, text=True, timeout=120)
     assert out.returncode == 0, out.stderr
     assert out.stdout.strip() == "1"
+
+
+_NOT_STATUS = {"cs_build_flags", "cs_param_tensor_count", "cs_destroy_model"}
+
+
+def test_every_entry_point_rejects_empty_arguments_on_the_host(b):
+    """Every call that returns a cs_status checks its pointers and sizes before any device
+    work: with null pointers and zero sizes it returns CS_ERR_ARG and leaves a message
+    (no GPU is touched, so this runs here)."""
+    import ctypes as C
+    zero = {C.c_int: 0, C.c_longlong: 0, C.c_size_t: 0, C.c_float: 0.0, C.c_double: 0.0}
+    checked = []
+    for name, (res, args) in b._SIGS.items():
+        if res is not C.c_int or name in _NOT_STATUS:
+            continue
+        call = [zero.get(a) for a in args]   # pointers of every kind -> None
+        st = getattr(b.lib, name)(*call)
+        assert st == b.CS_ERR_ARG, f"{name} returned {st}"
+        assert b.last_error(), name
+        checked.append(name)
+    assert len(checked) >= 25
+    # destroying a null model is a no-op, like free(NULL)
+    assert b.lib.cs_destroy_model(None) == b.CS_OK
