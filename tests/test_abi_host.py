@@ -111,3 +111,24 @@ def test_every_entry_point_rejects_empty_arguments_on_the_host(b):
     assert len(checked) >= 25
     # destroying a null model is a no-op, like free(NULL)
     assert b.lib.cs_destroy_model(None) == b.CS_OK
+
+
+def test_product_path_has_no_fallback():
+    """The package never imports the oracle, and its binding refuses to import without
+    the compiled library (no CPU or PyTorch fallback to fall back on)."""
+    import subprocess
+    import sys
+    pkg = os.path.join(ROOT, "paper_2607_23159_gb300")
+    for f in os.listdir(pkg):
+        if f.endswith(".py"):
+            src = open(os.path.join(pkg, f)).read()
+            assert not re.search(r"^\s*(from|import)\s+oracle\b", src, flags=re.M), f
+    code = ("import os, sys\n"
+            "real = os.path.exists\n"
+            "os.path.exists = lambda p: False if str(p).endswith('.so') else real(p)\n"
+            "try:\n"
+            "    import paper_2607_23159_gb300.binding\n"
+            "except ImportError as e:\n"
+            "    print('refused:', e)\n")
+    out = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, cwd=ROOT, timeout=120)
+    assert out.returncode == 0 and out.stdout.startswith("refused:") and "build" in out.stdout, out.stdout + out.stderr
