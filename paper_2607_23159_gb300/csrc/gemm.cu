@@ -11,24 +11,19 @@
 // loop of tile i+1.  Tiles are visited n-fastest so that the CTAs in flight share A
 // rows and the whole of B in L2.
 //
-// BN = 256 runs as clusters of two CTAs on vertically adjacent tiles with the same B tile.
-// MODE 2 (the default): rank 0 issues one M = 256 tcgen05.mma (cta_group::2) per K slice for
-// the pair; each CTA's shared memory holds its 128 A rows and half of the B tile, both
-// CTAs' TMA loads complete on rank 0's stage barrier, and the MMA commit releases the stage
-// in both CTAs.  MODE 1 keeps one MMA stream per CTA and multicasts each half of B to both.
+// BN = 256 runs as clusters of two CTAs on vertically adjacent tiles with the same B tile
+// (MODE 2): rank 0 issues one M = 256 tcgen05.mma (cta_group::2) per K slice for the pair;
+// each CTA's shared memory holds its 128 A rows and half of the B tile, both CTAs' TMA loads
+// complete on rank 0's stage barrier, and the MMA commit releases the stage in both CTAs.
 // Measured on GB300 (M 131040): the shared-memory writes of the B tile were the limit of
 // the single-CTA kernel; MODE 2 halves them (1.66 -> 1.83 PFLOP/s at N 8960, K 1536).
-// Every output element keeps the same K order in all modes.
+// Every output element keeps the same K order in both modes.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
 #include "common.cuh"
 #include "ptx.cuh"
 #include "tma_host.h"
-
-#ifndef CS_GEMM_PAIR_MODE
-#define CS_GEMM_PAIR_MODE 2   // the N >= 512 GEMMs: 1 = B multicast, 2 = two-SM MMA
-#endif
 
 namespace cs {
 
@@ -47,9 +42,9 @@ struct GemmArgs {
   int* err;
 };
 
-// MODE 0: one CTA per tile.  MODE 1: clusters of two, B multicast.  MODE 2: clusters of
-// two running one M = 256 tcgen05.mma (cta_group::2) per K slice: each CTA holds its 128 A
-// rows and half of the B tile, so every stage is half as large and the ring deeper.
+// MODE 0: one CTA per tile.  MODE 2: clusters of two running one M = 256 tcgen05.mma
+// (cta_group::2) per K slice: each CTA holds its 128 A rows and half of the B tile, so every
+// stage is half as large and the ring deeper.
 template <int BN, int MODE = 0>
 struct GemmCfg {
   static constexpr int BM = 128, BK = 64;
@@ -173,8 +168,9 @@ __global__ void __launch_bounds__(192, 1)
     gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmC, const GemmArgs p) {
   using Cfg = GemmCfg<BN, MODE>;
-  constexpr bool PAIR = MODE != 0;     // clusters of two CTAs on vertically adjacent tiles
+  static_assert(MODE == 0 || MODE == 2, "MODE 0 (one CTA per tile) or 2 (two-SM MMA)");
   constexpr bool TWO_SM = MODE == 2;   // one cta_group::2 MMA stream issued by the cluster's rank 0
+  constexpr bool PAIR = TWO_SM;        // clusters of two CTAs on vertically adjacent tiles
   constexpr int BM = Cfg::BM, BK = Cfg::BK, STAGES = Cfg::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -193,7 +189,7 @@ __global__ void __launch_bounds__(192, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], MODE == 1 ? 2 : 1);
+      mbar_init(&empty[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
@@ -214,7 +210,7 @@ __global__ void __launch_bounds__(192, 1)
   }
   tc_fence_before();
   block_sync();
-  if (PAIR) cluster_sync();   // the peer's barriers exist before anything is multicast into it
+  if (PAIR) cluster_sync();   // the peer's barriers exist before its loads complete on them
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -248,13 +244,9 @@ __global__ void __launch_bounds__(192, 1)
             tma_load_2d_2sm(sA + stage * Cfg::A_BYTES, &tmA, bar0, kb * BK, m0);
             tma_load_2d_2sm(sB + stage * Cfg::B_BYTES, &tmB, bar0, kb * BK, n0 + rank * (BN / 2));
           } else {
-            mbar_arrive_expect_tx(&full[stage], Cfg::STAGE_BYTES);   // MODE 1: half of B comes from the peer
+            mbar_arrive_expect_tx(&full[stage], Cfg::STAGE_BYTES);
             tma_load_2d(sA + stage * Cfg::A_BYTES, &tmA, &full[stage], kb * BK, m0);
-            if (PAIR)
-              tma_load_2d_mc(sB + stage * Cfg::B_BYTES + rank * (Cfg::B_BYTES / 2), &tmB, &full[stage], kb * BK,
-                             n0 + rank * (BN / 2), 0x3);
-            else
-              tma_load_2d(sB + stage * Cfg::B_BYTES, &tmB, &full[stage], kb * BK, n0);
+            tma_load_2d(sB + stage * Cfg::B_BYTES, &tmB, &full[stage], kb * BK, n0);
           }
           ++issued;
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
@@ -302,7 +294,6 @@ __global__ void __launch_bounds__(192, 1)
               umma_bf16_ss(d_tmem, sdesc_sw128(a0 + k * 32), sdesc_sw128(b0 + k * 32), Cfg::IDESC,
                            (kb | k) != 0 ? 1u : 0u);
           if constexpr (TWO_SM) umma_commit_2sm_mc(&empty[stage], 0x3);
-          else if constexpr (PAIR) umma_commit_mc(&empty[stage], 0x3);
           else umma_commit(&empty[stage]);
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
         }
@@ -447,7 +438,7 @@ __global__ void __launch_bounds__(192, 1)
 
   tc_fence_before();
   block_sync();
-  if (PAIR) cluster_sync();   // the peer has consumed everything this CTA multicast to it
+  if (PAIR) cluster_sync();   // the peer's MMAs and arrivals on this CTA's barriers are done
   if (warp == 1) {
     tc_fence_after();
     if constexpr (TWO_SM) tmem_dealloc_2sm(tmem_base, Cfg::TMEM_COLS);
@@ -458,7 +449,7 @@ __global__ void __launch_bounds__(192, 1)
 template <int BN, int EPI, int MODE>
 static cs_status launch_gemm(const void* A, const void* B, const GemmArgs& args, cudaStream_t stream) {
   using Cfg = GemmCfg<BN, MODE>;
-  constexpr bool PAIR = MODE != 0;
+  constexpr bool PAIR = MODE == 2;
   CUtensorMap ta, tb;
   const uint64_t da[2] = {(uint64_t)args.K, (uint64_t)args.M};
   const uint64_t sa[1] = {(uint64_t)args.K * 2};
@@ -528,7 +519,7 @@ static cs_status launch_gemm(const void* A, const void* B, const GemmArgs& args,
 
 template <int EPI>
 static cs_status dispatch_bn(const void* A, const void* B, const GemmArgs& args, cudaStream_t stream) {
-  if (args.N >= 512) return launch_gemm<256, EPI, CS_GEMM_PAIR_MODE>(A, B, args, stream);
+  if (args.N >= 512) return launch_gemm<256, EPI, 2>(A, B, args, stream);
   return launch_gemm<128, EPI, 0>(A, B, args, stream);
 }
 
