@@ -23,12 +23,15 @@ open are stated where they are used.
 Parity status: the cache rule, sampler, search and selection are pinned by closed
 forms and invariants in ``tests/test_oracle_pins.py``; each DiT primitive is pinned
 against textbook special cases, the block against an independent composition and the
-forward by token-permutation invariants.  The DiT forward as a whole has no printed value
-in the paper to pin against (parity unpinned as a whole; pinned per primitive).  The
-conditioning MLPs (timestep embedding to adaLN vectors, text projection) are conventions
-of the workload's architecture that nothing in the paper fixes: parity unpinned beyond
-their primitives.  ``tests/test_oracle_mutants.py`` checks that planted mistakes in the
-functions above fail the pins.
+forward by token-permutation invariants.  The conditioning MLPs (``DiT.modulation``:
+timestep sinusoid to the six adaLN vectors per block and the head's two;
+``DiT.text_kv``: text projection to per-block K/V) are pinned by closed-form values
+through identity weights (SiLU at +-ln 3, the odd/even identities of GELU), by the
+role each adaLN vector plays in the block and head, and by an independent torch.nn
+composition.  The DiT forward as a whole has no printed value in the paper to pin
+against (pinned per part and by invariants, not as a whole).
+``tests/test_oracle_mutants.py`` checks that planted mistakes in the functions above
+fail the pins.
 """
 from __future__ import annotations
 

@@ -40,6 +40,12 @@ BEAM = "test_beam_refill_layout_and_state_copy"
 BEAM_DEGENERATE = "test_beam_and_pruned_search_degenerate_cases"
 STEP = "test_search_step_equals_per_candidate_rollout"
 STATIC = "test_static_schedule_hand_example_and_every_one_is_uncached"
+MOD_CLOSED = "test_modulation_closed_form_through_identity_weights"
+MOD_SINUS = "test_modulation_sinusoid_path_closed_form"
+ADALN_ROLES = "test_adaln_vectors_play_their_roles_in_the_block"
+HEAD_ROLES = "test_head_modulation_roles"
+TEXT_CLOSED = "test_text_kv_closed_form_through_identity_weights"
+COND_TORCH = "test_conditioning_against_torch_nn_composition"
 
 # (id, oracle function, text replaced, replacement, pins that must fail on the mutant)
 MUTANTS = [
@@ -115,6 +121,33 @@ MUTANTS = [
     ("head-shift-scale-swapped", "DiT.velocity", "(1.0 + hm[1]) + hm[0]", "(1.0 + hm[0]) + hm[1]",
      [ZERO_BLOCKS]),
     ("head-without-norm", "DiT.velocity", "layer_norm(tok) * (1.0", "tok * (1.0", [ZERO_BLOCKS]),
+    ("block-shift-scale1-swapped", "DiT.block", "* (1.0 + scale1) + shift1", "* (1.0 + shift1) + scale1",
+     [ADALN_ROLES]),
+    ("block-shift-scale2-swapped", "DiT.block", "* (1.0 + scale2) + shift2", "* (1.0 + shift2) + scale2",
+     [ADALN_ROLES]),
+    ("block-gate2-dropped", "DiT.block", "x + gate2 * f", "x + f", [ADALN_ROLES]),
+    # conditioning MLPs (timestep embedding -> adaLN vectors; text projection -> K/V)
+    ("mod-silu-dropped", "DiT.modulation", 'linear(silu(e), p["mod_w"]', 'linear(e, p["mod_w"]',
+     [MOD_CLOSED, COND_TORCH]),
+    ("mod-shift-scale-swapped", "DiT.modulation", ".reshape(6, d)", ".reshape(6, d)[[1, 0, 2, 3, 4, 5]]",
+     [MOD_CLOSED, COND_TORCH]),
+    ("mod-offset-not-added", "DiT.modulation", 'm + p[f"blk{b}.mod_off"]', 'm + 0 * p[f"blk{b}.mod_off"]',
+     [MOD_CLOSED, COND_TORCH]),
+    ("mod-offset-of-block-0", "DiT.modulation", 'p[f"blk{b}.mod_off"]', 'p["blk0.mod_off"]',
+     [MOD_CLOSED, COND_TORCH]),
+    ("head-mod-silu-dropped", "DiT.modulation", "hm = linear(silu(e)", "hm = linear(e", [MOD_CLOSED, COND_TORCH]),
+    ("head-mod-shift-scale-swapped", "DiT.modulation", ".reshape(2, d)", ".reshape(2, d)[::-1]",
+     [MOD_CLOSED, HEAD_ROLES, COND_TORCH]),
+    ("time-mlp-silu-dropped", "DiT.modulation", "e = linear(silu(linear(timestep_sinusoid",
+     "e = linear((linear(timestep_sinusoid", [MOD_SINUS, COND_TORCH]),
+    ("sinusoid-time-scale", "timestep_sinusoid", "arg = 1000.0 * float(t)", "arg = float(t)",
+     [SINUS, MOD_SINUS, COND_TORCH]),
+    ("text-gelu-dropped", "DiT.text_kv", "txt = linear(gelu_tanh(linear(", "txt = linear((linear(",
+     [TEXT_CLOSED, COND_TORCH]),
+    ("text-kv-split-swapped", "DiT.text_kv", "kv.append((y[:, :d], y[:, d:]))", "kv.append((y[:, d:], y[:, :d]))",
+     [TEXT_CLOSED, COND_TORCH]),
+    ("text-kv-one-block", "DiT.text_kv", 'linear(txt, p[f"blk{b}.ckv_w"], p[f"blk{b}.ckv_b"])',
+     'linear(txt, p["blk0.ckv_w"], p["blk0.ckv_b"])', [TEXT_CLOSED, COND_TORCH]),
 ]
 
 

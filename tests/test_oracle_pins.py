@@ -344,6 +344,204 @@ def test_dit_zero_blocks_reduce_to_head_of_embedding():
     np.testing.assert_allclose(O.patchify(m.velocity(x, t, kv)), out, atol=1e-12)
 
 
+# ---------------------------------------------------- conditioning MLPs ---
+# The adaLN modulation MLP and the text projection are the workload architecture's
+# conditioning (Sec. 2 names a DiT conditioned on t and the text c; the block is fixed
+# by the workload).  Their pins: closed-form values through identity weights, the
+# roles of the six adaLN vectors and of the head's two inside the block, and an
+# independent torch.nn composition with every bias and offset non-zero.
+
+def _eye_stack(reps, d):
+    return np.concatenate([np.eye(d)] * reps, axis=0)
+
+
+def test_modulation_closed_form_through_identity_weights():
+    # time_w2 = 0 makes e = time_b2 exactly; with e = (ln 3, -ln 3, 0, ...) the SiLU
+    # has the closed forms SiLU(ln 3) = 3/4 ln 3, SiLU(-ln 3) = -1/4 ln 3, SiLU(0) = 0.
+    # mod_w / head_mod_w = stacked identities pass SiLU(e) to every vector, so chunk j
+    # of block b is SiLU(e) + b_mod[j] + offset_b[j] and the head's is SiLU(e) + b_hm[j].
+    cfg, m = _tiny_model(blocks=3)
+    d = cfg.d
+    rng = np.random.default_rng(21)
+    ln3 = math.log(3.0)
+    e0 = np.resize(np.array([ln3, -ln3, 0.0]), d)
+    silu_e0 = np.resize(np.array([0.75 * ln3, -0.25 * ln3, 0.0]), d)
+    m.p["time_w2"] = np.zeros((d, d))
+    m.p["time_b2"] = e0
+    m.p["mod_w"] = _eye_stack(6, d)
+    m.p["mod_b"] = rng.standard_normal(6 * d)
+    m.p["head_mod_w"] = _eye_stack(2, d)
+    m.p["head_mod_b"] = rng.standard_normal(2 * d)
+    for b in range(cfg.blocks):
+        m.p[f"blk{b}.mod_off"] = rng.standard_normal((6, d))
+    for t in (0.0, 0.3, 1.0):          # e does not depend on t here
+        mods, hm = m.modulation(t)
+        assert len(mods) == cfg.blocks
+        for b in range(cfg.blocks):
+            for j in range(6):         # shift1, scale1, gate1, shift2, scale2, gate2
+                np.testing.assert_allclose(mods[b][j], silu_e0 + m.p["mod_b"][j * d:(j + 1) * d]
+                                           + m.p[f"blk{b}.mod_off"][j], rtol=0, atol=1e-14)
+        for j in range(2):             # head shift, scale
+            np.testing.assert_allclose(hm[j], silu_e0 + m.p["head_mod_b"][j * d:(j + 1) * d], rtol=0, atol=1e-14)
+
+
+def test_modulation_sinusoid_path_closed_form():
+    # time_w1 = [I; 0], time_w2 = I and zero biases: e = SiLU(sinusoid(t)) on the first
+    # f_dim features and 0 after them; mod_w = stacked identities: every adaLN vector is
+    # SiLU(e).  At t = 0 the sinusoid is (1, ..., 1, 0, ..., 0), so the first half holds
+    # SiLU(SiLU(1)) with SiLU(1) = e/(e+1); at t = 1/2 its first cosine is cos(500).
+    cfg, m = _tiny_model(blocks=1)
+    d, f = cfg.d, cfg.f_dim
+    w1 = np.zeros((d, f))
+    w1[:f, :f] = np.eye(f)
+    m.p["time_w1"], m.p["time_b1"] = w1, np.zeros(d)
+    m.p["time_w2"], m.p["time_b2"] = np.eye(d), np.zeros(d)
+    m.p["mod_w"], m.p["mod_b"] = _eye_stack(6, d), np.zeros(6 * d)
+    m.p["blk0.mod_off"] = np.zeros((6, d))
+    silu = lambda z: z / (1.0 + math.exp(-z))
+    s1 = math.e / (math.e + 1.0)
+    mods, _ = m.modulation(0.0)
+    for j in range(6):
+        np.testing.assert_allclose(mods[0][j][:f // 2], silu(s1), rtol=1e-14)
+        np.testing.assert_array_equal(mods[0][j][f // 2:], 0.0)
+    mods, _ = m.modulation(0.5)
+    np.testing.assert_allclose(mods[0][0][0], silu(silu(math.cos(500.0))), rtol=1e-13)
+    np.testing.assert_allclose(mods[0][3][f // 2], silu(silu(math.sin(500.0))), rtol=1e-13)
+
+
+def _block_with(m, cfg, b, mod, zero):
+    for k in zero:
+        m.p[f"blk{b}.{k}"] = np.zeros_like(m.p[f"blk{b}.{k}"])
+    rng = np.random.default_rng(23)
+    x = rng.standard_normal((cfg.L, cfg.d))
+    kv = m.text_kv(synth.text_context(cfg))
+    return x, m.block(b, x, mod, kv[b])
+
+
+def test_adaln_vectors_play_their_roles_in_the_block():
+    # scale = -1 cancels the normalised input, leaving h = shift for every token; with
+    # the other branches' weights zero the block then adds the same vector to every
+    # token.  A gate of 0 removes its branch whatever the branch computes.
+    rng = np.random.default_rng(22)
+    cfg, m = _tiny_model(blocks=1)
+    d = cfg.d
+    mod = [rng.standard_normal(d) * 0.5 for _ in range(6)]
+    mod[1] = -np.ones(d)                                   # scale1
+    x, y = _block_with(m, cfg, 0, mod, ["cq_w", "co_w", "ff1_w", "ff2_w"])
+    r = y - x
+    np.testing.assert_allclose(r, np.broadcast_to(r[0], r.shape), atol=1e-12)
+    assert np.abs(r[0]).max() > 1e-3
+
+    cfg, m = _tiny_model(blocks=1)
+    mod = [rng.standard_normal(d) * 0.5 for _ in range(6)]
+    mod[4] = -np.ones(d)                                   # scale2
+    x, y = _block_with(m, cfg, 0, mod, ["qkv_w", "o_w", "cq_w", "co_w"])
+    r = y - x
+    np.testing.assert_allclose(r, np.broadcast_to(r[0], r.shape), atol=1e-12)
+    assert np.abs(r[0]).max() > 1e-3
+
+    # gates: with gate1 = gate2 = 0 the block is x + CA(LN(x)); random self-attention
+    # and FFN weights then change nothing
+    cfg, m = _tiny_model(blocks=1)
+    mod = [rng.standard_normal(d) * 0.5 for _ in range(6)]
+    mod[2] = np.zeros(d)
+    mod[5] = np.zeros(d)
+    kv = m.text_kv(synth.text_context(cfg))
+    x = rng.standard_normal((cfg.L, d))
+    y0 = m.block(0, x, mod, kv[0])
+    for k in ("qkv_w", "o_w", "ff1_w", "ff2_w"):
+        m.p[f"blk0.{k}"] = rng.standard_normal(m.p[f"blk0.{k}"].shape)
+    np.testing.assert_allclose(m.block(0, x, mod, kv[0]), y0, atol=1e-12)
+
+
+def test_head_modulation_roles():
+    # head scale = -1 (through head_mod_b, with head_mod_w = 0): every token's head
+    # input is the head shift, so the velocity is the same per-patch vector
+    # head_w shift + head_b at every token, for any latent
+    cfg, m = _tiny_model()
+    d = cfg.d
+    rng = np.random.default_rng(24)
+    shift = rng.standard_normal(d)
+    m.p["head_mod_w"] = np.zeros((2 * d, d))
+    m.p["head_mod_b"] = np.concatenate([shift, -np.ones(d)])
+    m.p["head_b"] = rng.standard_normal(cfg.P)
+    kv = m.text_kv(synth.text_context(cfg))
+    expect = m.p["head_w"] @ shift + m.p["head_b"]
+    for s in (0, 1):
+        x = synth.initial_noise(cfg, [s])[0].astype(np.float64)
+        v = O.patchify(m.velocity(x, 0.45, kv))
+        np.testing.assert_allclose(v, np.broadcast_to(expect, v.shape), atol=1e-12)
+
+
+def test_text_kv_closed_form_through_identity_weights():
+    # text_w1 = I, text_w2 = 2 I, text_b2 = beta, ckv_w = [I; 3 I]: per block b
+    #   K_b(c) = 2 GELU(c) + beta + kb_b,   V_b(c) = 3 (2 GELU(c) + beta) + vb_b.
+    # GELU(c) - GELU(-c) = c exactly (tanh form), and GELU(c) + GELU(-c) is within 2e-3
+    # of its exact-erf value c erf(c / sqrt 2).
+    cfg, m = _tiny_model(blocks=3)
+    d = cfg.d
+    assert cfg.d_text == d
+    rng = np.random.default_rng(25)
+    beta = rng.standard_normal(d)
+    m.p["text_w1"], m.p["text_b1"] = np.eye(d), np.zeros(d)
+    m.p["text_w2"], m.p["text_b2"] = 2.0 * np.eye(d), beta
+    for b in range(cfg.blocks):
+        m.p[f"blk{b}.ckv_w"] = np.concatenate([np.eye(d), 3.0 * np.eye(d)])
+        m.p[f"blk{b}.ckv_b"] = rng.standard_normal(2 * d)
+    c = rng.standard_normal((cfg.Lt, d)) * 1.5
+    kv_p, kv_m = m.text_kv(c), m.text_kv(-c)
+    even = c * np.vectorize(math.erf)(c / math.sqrt(2.0))     # GELU(c) + GELU(-c), exact-erf form
+    for b in range(cfg.blocks):
+        kb, vb = m.p[f"blk{b}.ckv_b"][:d], m.p[f"blk{b}.ckv_b"][d:]
+        (K, V), (Km, Vm) = kv_p[b], kv_m[b]
+        np.testing.assert_allclose(K - Km, 2.0 * c, atol=1e-12)
+        np.testing.assert_allclose(K + Km, 2.0 * even + 2.0 * (beta + kb), atol=4e-3)
+        np.testing.assert_allclose(V - 3.0 * K, np.broadcast_to(vb - 3.0 * kb, V.shape), atol=1e-12)
+
+
+def test_conditioning_against_torch_nn_composition():
+    """modulation() and text_kv() rebuilt from torch.nn.Linear modules, F.silu,
+    F.gelu(approximate='tanh') and a torch sinusoid with 10000^(-j/half) frequencies,
+    with every bias and offset random and non-zero."""
+    cfg, m = _tiny_model(blocks=2)
+    d, f = cfg.d, cfg.f_dim
+    rng = np.random.default_rng(26)
+    for k in list(m.p):
+        if k.endswith("_b") or k.endswith("_b1") or k.endswith("_b2") or k.endswith("mod_off"):
+            m.p[k] = rng.standard_normal(m.p[k].shape) * 0.3
+    T = lambda a: torch.from_numpy(np.asarray(a, np.float64))
+
+    def lin(wk, bk):
+        layer = torch.nn.Linear(m.p[wk].shape[1], m.p[wk].shape[0], dtype=torch.float64)
+        with torch.no_grad():
+            layer.weight.copy_(T(m.p[wk]))
+            layer.bias.copy_(T(m.p[bk]))
+        return layer
+
+    with torch.no_grad():
+        for t in (0.0, 0.37, 0.9):
+            half = f // 2
+            freq = torch.pow(torch.tensor(10000.0, dtype=torch.float64),
+                             -torch.arange(half, dtype=torch.float64) / half)
+            ang = (1000.0 * t) * freq
+            sinus = torch.cat([torch.cos(ang), torch.sin(ang)])
+            e = lin("time_w2", "time_b2")(TF.silu(lin("time_w1", "time_b1")(sinus)))
+            six = lin("mod_w", "mod_b")(TF.silu(e)).view(6, d)
+            head = lin("head_mod_w", "head_mod_b")(TF.silu(e)).view(2, d)
+            mods, hm = m.modulation(t)
+            for b in range(cfg.blocks):
+                np.testing.assert_allclose(np.asarray(mods[b]), (six + T(m.p[f"blk{b}.mod_off"])).numpy(),
+                                           atol=1e-12)
+            np.testing.assert_allclose(np.asarray(hm), head.numpy(), atol=1e-12)
+        ctx = T(synth.text_context(cfg))
+        txt = lin("text_w2", "text_b2")(TF.gelu(lin("text_w1", "text_b1")(ctx), approximate="tanh"))
+        kv = m.text_kv(synth.text_context(cfg))
+        for b in range(cfg.blocks):
+            k_t, v_t = lin(f"blk{b}.ckv_w", f"blk{b}.ckv_b")(txt).split(d, dim=1)
+            np.testing.assert_allclose(kv[b][0], k_t.numpy(), atol=1e-12)
+            np.testing.assert_allclose(kv[b][1], v_t.numpy(), atol=1e-12)
+
+
 # ------------------------------------------------------------ search variants ---
 
 def test_static_schedule_hand_example_and_every_one_is_uncached():
