@@ -6,10 +6,13 @@ none of the method's arithmetic (no model, no cache rule, no sampler).
 
 Recipe (every draw is a numpy ``Philox`` stream, key = the seed named below):
 
-* DiT weights: Xavier-uniform, ``U(-a, a)`` with ``a = sqrt(6 / (fan_in + fan_out))``,
-  rounded to the nearest bf16 value (round-half-even) so that a bf16 device copy
-  holds exactly the values the oracle sees.  Biases and the per-block modulation
-  offsets are 0.  One stream per parameter tensor, keyed ``(42, tensor index)``.
+* DiT weights: Xavier-uniform, ``U(-a, a)`` with ``a = sqrt(6 / (fan_in + fan_out))``
+  in float32.  By default each is rounded to the nearest bf16 value (round-half-even),
+  so that a bf16 device copy holds exactly the values the oracle sees and a parity
+  difference measures the kernels alone; ``round_bf16=False`` keeps the float32 draws,
+  which the library then rounds itself (parity then includes the weight rounding).
+  Biases and the per-block modulation offsets are 0.  One stream per parameter
+  tensor, keyed ``(42, tensor index)``.
 * Initial noise ``x_1`` of candidate ``i``: ``N(0, 1)`` float32 from key ``i``
   (the paper draws each candidate's noise from a generator seeded with the
   candidate's seed, Sec. Reproducibility).
@@ -153,7 +156,7 @@ def round_to_bf16(a: np.ndarray) -> np.ndarray:
     return u.view(np.float32)
 
 
-def _one_param(idx: int, shape, kind: str, seed: int, out: np.ndarray):
+def _one_param(idx: int, shape, kind: str, seed: int, out: np.ndarray, round_bf16: bool = True):
     if kind == "b":
         out[...] = 0.0
         return
@@ -161,11 +164,13 @@ def _one_param(idx: int, shape, kind: str, seed: int, out: np.ndarray):
     a = np.float32(np.sqrt(6.0 / (fan_in + fan_out)))
     g = np.random.Generator(np.random.Philox(key=[seed, idx]))
     u = g.random(out.size, dtype=np.float32)
-    out[...] = round_to_bf16((u * np.float32(2.0) - np.float32(1.0)) * a).reshape(shape)
+    w = (u * np.float32(2.0) - np.float32(1.0)) * a
+    out[...] = (round_to_bf16(w) if round_bf16 else w).reshape(shape)
 
 
-def make_params(m: ModelConfig, seed: int = WEIGHT_SEED, threads: int | None = None):
-    """All DiT parameters as (flat float32 buffer, {name: view into it})."""
+def make_params(m: ModelConfig, seed: int = WEIGHT_SEED, threads: int | None = None, round_bf16: bool = True):
+    """All DiT parameters as (flat float32 buffer, {name: view into it}); weights rounded
+    to bf16 values unless ``round_bf16`` is False."""
     lay = param_layout(m)
     flat = np.empty(param_count(m), dtype=np.float32)
     views, off = {}, 0
@@ -176,7 +181,7 @@ def make_params(m: ModelConfig, seed: int = WEIGHT_SEED, threads: int | None = N
     jobs = [(i, s, k, views[n]) for i, (n, s, k) in enumerate(lay)]
     nthr = threads or min(16, os.cpu_count() or 1)
     with ThreadPoolExecutor(nthr) as ex:
-        list(ex.map(lambda j: _one_param(j[0], j[1], j[2], seed, j[3]), jobs))
+        list(ex.map(lambda j: _one_param(j[0], j[1], j[2], seed, j[3], round_bf16), jobs))
     return flat, views
 
 

@@ -6,6 +6,8 @@
   error, top-1 identical);
 * the 1.3B model width (d 1536, 12 x 128 heads, FFN 8960, 512 x 4096 text) with 2 blocks
   on a small latent, where the oracle still finishes in seconds;
+* both with bf16-valued weights (the kernels alone) and with unrounded float32 weights
+  that the library rounds on load (bf16 vs fp32, the weight rounding included);
 * properties that hold at any size: batch invariance (a candidate's result is bitwise
   the same alone or inside any batch), run-to-run determinism, tau = 0 equals always
   computing, and the closed form of an all-skip rollout.
@@ -33,9 +35,9 @@ def dev(a, dtype=torch.float32):
 
 
 class Inputs:
-    def __init__(self, m, N, seeds=None):
+    def __init__(self, m, N, seeds=None, round_bf16=True):
         self.m = m
-        self.flat, self.params = synth.make_params(m)
+        self.flat, self.params = synth.make_params(m, round_bf16=round_bf16)
         self.ctx = synth.text_context(m)
         self.x1 = synth.initial_noise(m, seeds if seeds is not None else range(N))
         self.y = synth.target_latent(m)
@@ -101,6 +103,18 @@ def tiny():
     return cfg, inp, ref
 
 
+@pytest.fixture(scope="module")
+def tiny_fp32():
+    """The tiny workload with unrounded float32 weights: the oracle takes them as they
+    are and the library rounds them to bf16 on load, so the parity includes the weight
+    rounding (bf16 vs fp32)."""
+    cfg = synth.CONFIGS["tiny"]
+    inp = Inputs(cfg.model, cfg.N, round_bf16=False)
+    assert not np.array_equal(inp.flat, synth.round_to_bf16(inp.flat))
+    ref = oracle_search(inp, cfg.N, cfg.T, cfg.tau, cfg.K_w, cfg.K_c)
+    return cfg, inp, ref
+
+
 def test_tiny_dit_forward_matches_oracle_on_compacted_subset(B, tiny):
     cfg, inp, _ = tiny
     m = inp.m
@@ -122,8 +136,9 @@ def test_tiny_dit_forward_matches_oracle_on_compacted_subset(B, tiny):
     model.close()
 
 
-def test_tiny_search_free_running_matches_oracle(B, tiny):
-    cfg, inp, (xo, mo, so, pres) = tiny
+@pytest.mark.parametrize("weights", ["bf16-valued", "fp32"])
+def test_tiny_search_free_running_matches_oracle(B, tiny, tiny_fp32, weights):
+    cfg, inp, (xo, mo, so, pres) = tiny if weights == "bf16-valued" else tiny_fp32
     st, mg, sg, _ = gpu_search(B, inp, cfg.N, cfg.T, cfg.tau, cfg.K_w, cfg.K_c)
     for k in range(cfg.T):
         diff = mg[k] != mo[k]
@@ -137,8 +152,9 @@ def test_tiny_search_free_running_matches_oracle(B, tiny):
     assert int(np.argmax(sg)) == int(O.topk(so, 1)[0])
 
 
-def test_tiny_search_mask_replay_matches_oracle(B, tiny):
-    cfg, inp, (xo, mo, so, _) = tiny
+@pytest.mark.parametrize("weights", ["bf16-valued", "fp32"])
+def test_tiny_search_mask_replay_matches_oracle(B, tiny, tiny_fp32, weights):
+    cfg, inp, (xo, mo, so, _) = tiny if weights == "bf16-valued" else tiny_fp32
     st, mg, sg, _ = gpu_search(B, inp, cfg.N, cfg.T, cfg.tau, cfg.K_w, cfg.K_c, force_masks=~mo)
     assert np.array_equal(mg, mo)
     g = st["x"].cpu().numpy().reshape(xo.shape)
@@ -151,10 +167,11 @@ def test_tiny_search_mask_replay_matches_oracle(B, tiny):
 
 # --------------------------------------------------- 1.3B width, small latent ----
 
-def test_wan13b_width_small_latent_matches_oracle(B):
+@pytest.mark.parametrize("round_bf16", [True, False])
+def test_wan13b_width_small_latent_matches_oracle(B, round_bf16):
     m = synth.replace_model(synth.WAN_1_3B, F=2, H=16, W=16, blocks=2)
     N, T, tau = 2, 3, 0.1
-    inp = Inputs(m, N)
+    inp = Inputs(m, N, round_bf16=round_bf16)
     xo, mo, so, _ = oracle_search(inp, N, T, tau, 1, 1)
     st, mg, sg, _ = gpu_search(B, inp, N, T, tau, 1, 1, force_masks=~mo)
     g = st["x"].cpu().numpy().reshape(xo.shape)
