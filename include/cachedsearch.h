@@ -154,7 +154,9 @@ cs_status cs_cache_decide(const float* x_dev, const float* x_ref_dev, float* acc
  *   Limits: N <= CS_NOALLOC_MAX_N candidates and D <= CS_NOALLOC_MAX_CHUNKS * 8192
  *   elements per candidate; larger sizes return CS_ERR_ARG with a message, nothing runs.
  *   The first call on a device looks up the array's device address (cudaGetSymbolAddress)
- *   with that device current; make that first call before any stream capture.
+ *   with that device current; make that first call before any stream capture.  The
+ *   address is kept for the life of the process: after cudaDeviceReset on that device
+ *   it would be stale, so a process that resets a device must not call this again.
  *   All calls on a device share the array: calls that overlap on the GPU (other streams
  *   or threads) race and must be serialised by the caller.  Each call writes every
  *   partial it reads, so nothing from a previous call needs clearing.
@@ -241,7 +243,8 @@ cs_status cs_search_step_host(cs_model* model, float* x_host, float* x_ref_dev, 
                               float t_next, float tau, int K_w, int K_c, uint8_t* skip_mask_host,
                               int* n_computed, cudaStream_t stream);
 
-/* scores_dev[i] = -||x_i - target||_2 (the verifier stand-in, Algorithm 1 "r_i <- V(y_i, c)"). */
+/* scores_dev[i] = -||x_i - target||_2: the stand-in for the verifier score that Algorithm 1
+ * assigns to each explored candidate. */
 cs_status cs_score(const float* x_dev, const float* target_dev, int N, long long D, float* scores_dev,
                    void* workspace_dev, cudaStream_t stream);
 

@@ -871,7 +871,9 @@ constexpr int kStaticMaxChunks = CS_NOALLOC_MAX_CHUNKS;
 static __device__ __align__(256) float g_decide_scratch[kStaticMaxN * kStaticMaxChunks * 2];
 
 static std::mutex g_scratch_mu;
-static float* g_scratch_ptr[256] = {};   // device address of g_decide_scratch, per device ordinal
+// Device address of g_decide_scratch per device ordinal, looked up once and kept for the
+// life of the process (a cudaDeviceReset would leave it stale; the header says so).
+static float* g_scratch_ptr[256] = {};
 
 // Device address of the scratch array on the current device (looked up once per device).
 static cs_status static_scratch(float** out) {
