@@ -194,6 +194,38 @@ class DiT:
                    p[f"blk{b}.ff2_w"], p[f"blk{b}.ff2_b"])
         return x + gate2 * f
 
+    def block_rows(self, b, x, rows, mod, kv):
+        """The block's output for the token rows ``rows`` only, x [L, d] being every token
+        of the input.  Attention is the only step that mixes tokens, and it does so through
+        the keys and values alone: K and V come from every row of x, everything else (the
+        queries, projections, cross-attention, FFN) from the selected rows, so each selected
+        row equals the same row of :meth:`block`."""
+        p, H, d = self.p, self.cfg.heads, self.cfg.d
+        shift1, scale1, gate1, shift2, scale2, gate2 = mod
+        kv_self = linear(layer_norm(x) * (1.0 + scale1) + shift1, p[f"blk{b}.qkv_w"][d:], p[f"blk{b}.qkv_b"][d:])
+        xr = x[rows]
+        q = linear(layer_norm(xr) * (1.0 + scale1) + shift1, p[f"blk{b}.qkv_w"][:d], p[f"blk{b}.qkv_b"][:d])
+        sa = multi_head_attention(q, kv_self[:, :d], kv_self[:, d:], H)
+        xr = xr + gate1 * linear(sa, p[f"blk{b}.o_w"], p[f"blk{b}.o_b"])
+        qc = linear(layer_norm(xr), p[f"blk{b}.cq_w"], p[f"blk{b}.cq_b"])
+        xr = xr + linear(multi_head_attention(qc, kv[0], kv[1], H), p[f"blk{b}.co_w"], p[f"blk{b}.co_b"])
+        h = layer_norm(xr) * (1.0 + scale2) + shift2
+        f = linear(gelu_tanh(linear(h, p[f"blk{b}.ff1_w"], p[f"blk{b}.ff1_b"])), p[f"blk{b}.ff2_w"], p[f"blk{b}.ff2_b"])
+        return xr + gate2 * f
+
+    def velocity_rows(self, x, t, kv, rows):
+        """Velocity of a one-block model at the token rows ``rows``, in token layout
+        [len(rows), 4C] (feature ``4c + 2 ph + pw`` of token l, as :func:`patchify`): the
+        rows of ``patchify(velocity(x, t, kv))``.  Only the last block may be evaluated on
+        a subset of rows, so the model must have exactly one block."""
+        if self.cfg.blocks != 1:
+            raise ValueError("velocity_rows needs a one-block model (the next block would need every row)")
+        mods, hm = self.modulation(t)
+        tok = linear(patchify(np.asarray(x, np.float64)), self.p["patch_w"], self.p["patch_b"])
+        out = self.block_rows(0, tok, rows, mods[0], kv[0])
+        h = layer_norm(out) * (1.0 + hm[1]) + hm[0]
+        return linear(h, self.p["head_w"], self.p["head_b"])
+
     def velocity(self, x, t, kv):
         """v_theta(x, t, c) for one latent x [C, F, H, W] -> [C, F, H, W]."""
         c = self.cfg

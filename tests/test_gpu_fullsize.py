@@ -159,3 +159,41 @@ def test_full_size_fused_cache_step_every_element(B):
     for i in (1, 3):    # computed: the reference and the transformation vector are refreshed
         np.testing.assert_array_equal(st["x_ref"][i].cpu().numpy(), x[i])
         np.testing.assert_allclose(st["delta"][i].cpu().numpy(), v[i] - x[i], rtol=1e-6, atol=1e-6)
+
+
+def test_composed_block_and_head_full_length_sampled_rows(B):
+    """The composed DiT forward (patch embed, LayerNorm + adaLN, QKV scatter, self-attention
+    over all 32760 tokens, gated O projection, cross-attention to the 512 text tokens, GELU
+    FFN, head) of one 1.3B-width block on a compacted subset of 4 candidates (idx 0, 2, 3),
+    against the oracle's one-block velocity on 40 sampled token rows x all 64 features;
+    full-length K/V on both sides.  The row outside the subset stays untouched."""
+    m = synth.replace_model(synth.WAN_1_3B, blocks=1)
+    flat, params = synth.make_params(m)
+    ctx = synth.text_context(m)
+    x1 = synth.initial_noise(m, range(NC))
+    model = B.Model(m, NC)
+    model.load_weights(flat)
+    model.set_text_context(dev(ctx))
+    x = dev(x1.reshape(NC, -1))
+    v = torch.full((NC, m.D), 7.0, device="cuda")
+    idx = torch.tensor([0, 2, 3], dtype=torch.int32, device="cuda")
+    t = 0.7
+    model.dit_forward(x, idx, 3, t, v)
+    torch.cuda.synchronize()
+    assert model.device_error() == 0
+    model.close()
+    got = v.cpu().numpy()
+    assert np.all(got[1] == 7.0)
+    dit = O.DiT(m, params)
+    kv = dit.text_kv(ctx)
+    rng = np.random.default_rng(71)
+    rows = np.unique(np.concatenate([rng.integers(0, m.L, 38), [0, m.L - 1]]))
+    f_, hh, ww = rows // ((m.H // 2) * (m.W // 2)), (rows // (m.W // 2)) % (m.H // 2), rows % (m.W // 2)
+    for i in (0, 2, 3):
+        ref = dit.velocity_rows(x1[i], t, kv, rows)                      # [rows, 4C]
+        g = got[i].reshape(m.C, m.F, m.H, m.W)
+        # token layout of the GPU velocity at the sampled rows: feature 4c + 2 ph + pw
+        gt = np.stack([g[c, f_, 2 * hh + ph, 2 * ww + pw] for c in range(m.C) for ph in (0, 1) for pw in (0, 1)],
+                      axis=1)
+        rel = np.abs(gt - ref).max() / np.abs(ref).max()
+        assert rel < 2e-2, (i, rel)

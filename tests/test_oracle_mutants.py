@@ -46,6 +46,7 @@ ADALN_ROLES = "test_adaln_vectors_play_their_roles_in_the_block"
 HEAD_ROLES = "test_head_modulation_roles"
 TEXT_CLOSED = "test_text_kv_closed_form_through_identity_weights"
 COND_TORCH = "test_conditioning_against_torch_nn_composition"
+ROWS = "test_row_subset_forms_equal_the_full_forward"
 
 # (id, oracle function, text replaced, replacement, pins that must fail on the mutant)
 MUTANTS = [
@@ -146,6 +147,11 @@ MUTANTS = [
      [TEXT_CLOSED, COND_TORCH]),
     ("text-kv-split-swapped", "DiT.text_kv", "kv.append((y[:, :d], y[:, d:]))", "kv.append((y[:, d:], y[:, :d]))",
      [TEXT_CLOSED, COND_TORCH]),
+    ("rows-keys-from-subset", "DiT.block_rows", "kv_self = linear(layer_norm(x) *", "kv_self = linear(layer_norm(x[rows]) *",
+     [ROWS]),
+    ("rows-value-heads-from-keys", "DiT.block_rows", "kv_self[:, :d], kv_self[:, d:], H)",
+     "kv_self[:, :d], kv_self[:, :d], H)", [ROWS]),
+    ("rows-head-scale-dropped", "DiT.velocity_rows", "* (1.0 + hm[1]) + hm[0]", "+ hm[0]", [ROWS]),
     ("text-kv-one-block", "DiT.text_kv", 'linear(txt, p[f"blk{b}.ckv_w"], p[f"blk{b}.ckv_b"])',
      'linear(txt, p["blk0.ckv_w"], p["blk0.ckv_b"])', [TEXT_CLOSED, COND_TORCH]),
 ]

@@ -344,6 +344,27 @@ def test_dit_zero_blocks_reduce_to_head_of_embedding():
     np.testing.assert_allclose(O.patchify(m.velocity(x, t, kv)), out, atol=1e-12)
 
 
+def test_row_subset_forms_equal_the_full_forward():
+    # the block and the one-block velocity evaluated on a subset of token rows are the
+    # same rows of the full evaluation (attention mixes tokens only through K and V)
+    cfg, m = _tiny_model(blocks=1)
+    rng = np.random.default_rng(27)
+    for k in list(m.p):
+        if k.endswith("_b") or k.endswith("mod_off"):
+            m.p[k] = rng.standard_normal(m.p[k].shape) * 0.3
+    kv = m.text_kv(synth.text_context(cfg))
+    mods, _ = m.modulation(0.55)
+    x = rng.standard_normal((cfg.L, cfg.d))
+    rows = np.array([0, 5, 17, cfg.L - 1])
+    np.testing.assert_allclose(m.block_rows(0, x, rows, mods[0], kv[0]), m.block(0, x, mods[0], kv[0])[rows],
+                               atol=1e-11)
+    lat = synth.initial_noise(cfg, [3])[0].astype(np.float64)
+    np.testing.assert_allclose(m.velocity_rows(lat, 0.55, kv, rows), O.patchify(m.velocity(lat, 0.55, kv))[rows],
+                               atol=1e-11)
+    with pytest.raises(ValueError):
+        _tiny_model(blocks=2)[1].velocity_rows(lat, 0.5, kv, rows)
+
+
 # ---------------------------------------------------- conditioning MLPs ---
 # The adaLN modulation MLP and the text projection are the workload architecture's
 # conditioning (Sec. 2 names a DiT conditioned on t and the text c; the block is fixed
