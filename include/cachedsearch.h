@@ -205,14 +205,16 @@ cs_status cs_search_step_cfg(cs_model* model, float* x_dev, float* x_ref_dev, fl
                              cudaStream_t stream);
 
 /* Single-pass form used by cs_search_step.  cs_cache_decide_skip takes the decision of
- * every candidate (as cs_cache_decide) and, in the same launch, applies Eq. skip + Eq.
- * euler to the skipped ones (and writes their score partials if target_dev is given), so
- * a skipped candidate's x, x_ref and Delta are read once and x written once.  One
- * cooperative launch with a bounded grid barrier; needs D % 4 == 0, 16-byte aligned
- * tensors and cs_cache_workspace_bytes(N, D) of workspace (its barrier words are reset
- * by the call).  cs_cache_apply_computed then updates only the computed candidates
- * (Eq. delta + Eq. euler, v_dev from the DiT) and, with target_dev, finalises the scores
- * of all candidates. */
+ * every candidate (as cs_cache_decide, with the same arithmetic and results) and applies
+ * Eq. skip + Eq. euler to the skipped ones (writing their score partials if target_dev
+ * is given), so that a skipped candidate's x_ref and Delta are read once, x read while
+ * still in L2 and written once.  Two launches and no grid-wide wait: the drift pass,
+ * in which the CTA that completes a candidate's last chunk decides it, then the skip
+ * update, scheduled by programmatic dependent launch while the first drains.  Needs
+ * D % 8 == 0, 32-byte aligned tensors and cs_cache_workspace_bytes(N, D) of workspace
+ * (its arrival counters are cleared by the call).  cs_cache_apply_computed then updates
+ * only the computed candidates (Eq. delta + Eq. euler, v_dev from the DiT) and, with
+ * target_dev, finalises the scores of all candidates. */
 cs_status cs_cache_decide_skip(float* x_dev, const float* x_ref_dev, const float* delta_dev, float* accum_dev,
                                uint8_t* has_ref_dev, int N, long long D, int step_k, int T, float t_cur,
                                float t_next, float tau, int K_w, int K_c, const uint8_t* force_compute_dev,
@@ -223,13 +225,36 @@ cs_status cs_cache_apply_computed(float* x_dev, float* x_ref_dev, float* delta_d
                                   const float* target_dev, float* scores_dev, void* workspace_dev,
                                   cudaStream_t stream);
 
+/* The computed candidates' update taken directly from the DiT head's output in token
+ * layout (the unpatchify scatter fused with Eq. delta and Eq. euler), so that the
+ * velocity is never written to memory as a latent.  For j < n_c, candidate i = idx[j]
+ * and latent element (c, f, h, w) of a [C][F][H][W] latent:
+ *   v = hout[(j*L + l)*4C + 4c + 2(h%2) + (w%2)],  l = (f*(H/2) + h/2)*(W/2) + w/2,
+ *   Delta_i = v - x_i;  x_ref_i = x_i;  x_i += (t_next - t_cur) v;
+ *   accum[i] = 0, has_ref[i] = 1, skip_mask[i] = 0.
+ * hout_dev: float32 [n_c * L][4C] (the head Linear's output rows of the compacted batch).
+ * Needs even H, W % 4 == 0 and 16-byte aligned tensors.  With target_dev, the computed
+ * candidates' score partials go to tile_partials_dev (float32 [N][F*H/2]) and
+ * scores_dev[i] = -||x0_i - target||_2 is finalised for all N candidates, the skipped
+ * ones from the partials cs_cache_decide_skip left in workspace_dev (same target). */
+cs_status cs_cache_apply_tokens(float* x_dev, float* x_ref_dev, float* delta_dev, float* accum_dev,
+                                uint8_t* has_ref_dev, uint8_t* skip_mask_dev, const float* hout_dev,
+                                const int32_t* compute_idx_dev, int n_c, int N, int C, int F, int H, int W,
+                                float t_cur, float t_next, const float* target_dev, float* scores_dev,
+                                void* workspace_dev, float* tile_partials_dev, int* err_dev, cudaStream_t stream);
+
 /* One denoising step of N candidates (the unit of work of the search):
- * cs_cache_decide_skip, then cs_dit_forward on the computing subset, then
- * cs_cache_apply_computed.
+ * cs_cache_decide_skip, then the DiT forward (as cs_dit_forward) on the computing
+ * subset, then the computed candidates' update from the head's token output
+ * (cs_cache_apply_tokens; latents with W % 4 != 0 take the velocity scatter and
+ * cs_cache_apply_computed instead).
  * State buffers (x, x_ref, delta: [N][D]; accum: [N]; has_ref: [N]) are caller-owned
  * device memory and are updated in place; a fresh search starts with has_ref = 0.
  * Synchronises once to read the number of computing candidates; that count is returned
- * in *n_computed (host, nullable). */
+ * in *n_computed (host, nullable).  A warm-up or cool-down step without a forced mask
+ * computes every candidate (Sec. 3.1): it takes no decision pass and does not
+ * synchronise, so a device error recorded during it is returned by the next call that
+ * synchronises (a free step, cs_search_step_host or cs_device_error). */
 cs_status cs_search_step(cs_model* model, float* x_dev, float* x_ref_dev, float* delta_dev, float* accum_dev,
                          uint8_t* has_ref_dev, int N, int step_k, int T, float t_cur, float t_next, float tau,
                          int K_w, int K_c, const uint8_t* force_compute_dev, uint8_t* skip_mask_dev,

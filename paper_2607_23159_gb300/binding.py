@@ -65,6 +65,7 @@ _SIGS = {
     "cs_cache_apply": (I, [P, P, P, P, P, I, LL, F, F, P, P, P, P]),
     "cs_cache_decide_skip": (I, [P, P, P, P, P, I, LL, I, I, F, F, F, I, I, P, P, P, P, P, P, P, P]),
     "cs_cache_apply_computed": (I, [P, P, P, P, P, I, LL, F, F, P, P, P, P]),
+    "cs_cache_apply_tokens": (I, [P, P, P, P, P, P, P, P, I, I, I, I, I, I, F, F, P, P, P, P, P, P]),
     "cs_search_step": (I, [P, P, P, P, P, P, I, I, I, F, F, F, I, I, P, P, P, P, P, P]),
     "cs_search_step_host": (I, [P, P, P, P, P, P, I, I, I, F, F, F, I, I, P, P, P]),
     "cs_score": (I, [P, P, I, LL, P, P, P]),
@@ -179,6 +180,17 @@ def cache_decide_noalloc(x, x_ref, accum, has_ref, step_k, T, tau, K_w, K_c, ski
     check(lib.cs_cache_decide_noalloc(_ptr(x), _ptr(x_ref), _ptr(accum), _ptr(has_ref), N, Dn, step_k, T, tau, K_w,
                                       K_c, _ptr(force), _ptr(skip_mask), _ptr(compute_idx), _ptr(n_compute),
                                       _ptr(err), _stream(stream)))
+
+
+def cache_apply_tokens(st, skip_mask, hout, compute_idx, n_c, C, F, H, W, t_cur, t_next, workspace=None,
+                       target=None, scores=None, tile_partials=None, err=None, stream=None):
+    """cs_cache_apply_tokens: the computed candidates' update from the head's token output
+    ``hout`` [n_c * L, 4C] (state dict ``st`` as from :func:`new_state`)."""
+    N = st["x"].shape[0]
+    check(lib.cs_cache_apply_tokens(_ptr(st["x"]), _ptr(st["x_ref"]), _ptr(st["delta"]), _ptr(st["accum"]),
+                                    _ptr(st["has_ref"]), _ptr(skip_mask), _ptr(hout), _ptr(compute_idx), n_c, N, C,
+                                    F, H, W, t_cur, t_next, _ptr(target), _ptr(scores), _ptr(workspace),
+                                    _ptr(tile_partials), _ptr(err), _stream(stream)))
 
 
 def cache_apply(x, x_ref, delta, v, skip_mask, t_cur, t_next, workspace=None, target=None, scores=None,

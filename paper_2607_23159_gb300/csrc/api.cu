@@ -54,6 +54,11 @@ struct cs_model {
   bf16 *tok, *hbuf, *obuf, *q, *k, *vt, *fbuf;
   float *resid, *hout, *cond_scratch, *mods, *hmod, *v, *x_host_stage;
   int32_t *idx, *n_compute;
+  int32_t* idx_all;   // 0, 1, ..., max_batch - 1: the compaction list of an all-compute step
+  unsigned* cache_counters;   // arrival counters [max_batch + 1] (zero between steps)
+  uint8_t* cache_dec;         // decisions [max_batch]
+  float* tpart;       // score partials of computed candidates per token row [max_batch][F*H/2]
+  bool tokens_update = false;   // computed update straight from the head's token output
   uint8_t* skip_tmp;
   void* cache_ws;
   int* err;
@@ -246,6 +251,10 @@ extern "C" cs_status cs_init_model(const cs_model_config* cfg, cs_model** out) {
   addf(&m->v, (size_t)cfg->max_batch * m->D);
   addf(&m->x_host_stage, (size_t)cfg->max_batch * m->D);
   items.push_back({reinterpret_cast<void**>(&m->idx), (size_t)cfg->max_batch * 4});
+  items.push_back({reinterpret_cast<void**>(&m->idx_all), (size_t)cfg->max_batch * 4});
+  items.push_back({reinterpret_cast<void**>(&m->cache_counters), (size_t)(cfg->max_batch + 1) * 4});
+  items.push_back({reinterpret_cast<void**>(&m->cache_dec), (size_t)cfg->max_batch});
+  addf(&m->tpart, (size_t)cfg->max_batch * cfg->F * (cfg->H / 2));
   items.push_back({reinterpret_cast<void**>(&m->n_compute), 16});
   items.push_back({reinterpret_cast<void**>(&m->skip_tmp), (size_t)cfg->max_batch});
   items.push_back({&m->cache_ws, cs_cache_workspace_bytes(cfg->max_batch, m->D)});
@@ -266,7 +275,11 @@ extern "C" cs_status cs_init_model(const cs_model_config* cfg, cs_model** out) {
     *it.dst = static_cast<char*>(m->ws) + off;
     off += it.bytes;
   }
-  cudaMemset(m->ws, 0, total);   // Q/K head-dim padding must read as zero
+  cudaMemset(m->ws, 0, total);   // Q/K head-dim padding and the cache step's counters start at zero
+  std::vector<int32_t> iota(cfg->max_batch);
+  for (int i = 0; i < cfg->max_batch; ++i) iota[i] = i;
+  cudaMemcpy(m->idx_all, iota.data(), iota.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
+  m->tokens_update = cs::apply_tokens_supported(cfg->C, cfg->F, cfg->H, cfg->W);
   std::vector<float*> offs(nb);
   for (size_t b = 0; b < nb; ++b) offs[b] = m->blk[b].mod_off;
   cudaMemcpy(m->mod_offs_dev, offs.data(), nb * sizeof(float*), cudaMemcpyHostToDevice);
@@ -449,6 +462,7 @@ extern "C" cs_status cs_set_null_text_context(cs_model* m, const float* ctx, cud
 // idx[j] / x_rows (kv_sets = 2 for guidance), velocity written to v[idx[j]].
 static cs_status dit_forward_impl(cs_model* m, const float* x, const int32_t* idx, int n_c, int x_rows, int kv_sets,
                                   float t, float* v, cudaStream_t s) {
+  // v == nullptr: stop after the head Linear; the velocity rows stay in m->hout (token layout)
   if (n_c == 0) return CS_OK;
   const cs_model_config& c = m->cfg;
   const int d = c.d, L = m->L, M = n_c * L;
@@ -494,6 +508,7 @@ static cs_status dit_forward_impl(cs_model* m, const float* x, const int32_t* id
   CS_TRY(cs::layernorm_modulate(m->resid, m->hmod, m->hmod + d, m->hbuf, M, d, s));
   CS_TRY(record_end(m, 4, s, ev, 0.0));
   CS_TRY(gemm(m, m->hbuf, m->head_w, CS_EPI_F32, m->head_b, nullptr, m->hout, m->P, M, m->P, d, s));
+  if (!v) return CS_OK;
   CS_TRY(record_begin(m, 4, s, ev));
   CS_TRY(cs::unpatchify(m->hout, idx, n_c, c.C, c.F, c.H, c.W, v, idx_limit, m->err, s));
   CS_TRY(record_end(m, 4, s, ev, 0.0));
@@ -516,32 +531,49 @@ static cs_status step_impl(cs_model* m, float* x, float* x_ref, float* delta, fl
   CS_REQUIRE(m && x && x_ref && delta && accum && has_ref && skip, "cs_search_step: null pointer");
   CS_REQUIRE(N > 0 && N <= m->cfg.max_batch, "cs_search_step: N=%d outside 1..max_batch=%d", N, m->cfg.max_batch);
   CS_REQUIRE(!target || scores, "cs_search_step: scoring needs scores");
+  CS_REQUIRE(k >= 1 && k <= T, "cs_search_step: step %d outside 1..T=%d", k, T);
   const long long D = m->D;
+  const cs_model_config& c = m->cfg;
   cudaEvent_t ev[2];
   const bool wf = k <= K_w || k > T - K_c;
-  CS_TRY(record_begin(m, 3, s, ev));
-  // decision + the update of skipped candidates in one pass; computed ones after the DiT
-  CS_TRY(cs_cache_decide_skip(x, x_ref, delta, accum, has_ref, N, D, k, T, t_cur, t_next, tau, K_w, K_c, force, skip,
-                              m->idx, m->n_compute, target, m->cache_ws, m->err, s));
-  CS_TRY(record_end(m, 3, s, ev, 0.0));
-  CS_CUDA(cudaMemcpyAsync(m->n_host, m->n_compute, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
-  CS_CUDA(cudaMemcpyAsync(m->n_host + 1, m->err, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
-  CS_CUDA(cudaStreamSynchronize(s));
-  const int n_c = m->n_host[0];
-  if (m->n_host[1] != 0) {
-    cs::set_error("cs_search_step: device error %d recorded before step %d", m->n_host[1], k);
-    const int code = m->n_host[1];
-    cudaMemsetAsync(m->err, 0, sizeof(int), s);
-    return (cs_status)code;
+  const bool tokens = m->tokens_update;
+  int n_c = N;
+  const int32_t* idx = m->idx;
+  if (tokens && wf && !force) {
+    // warm-up / cool-down: every candidate computes and no drift is evaluated (Sec. 3.1);
+    // the computed update below writes the state (a = 0, has_ref = 1, skip = 0)
+    idx = m->idx_all;
+  } else {
+    // decisions + the update of skipped candidates; computed ones after the DiT
+    CS_TRY(record_begin(m, 3, s, ev));
+    CS_TRY(cs::decide_skip_run(x, x_ref, delta, accum, has_ref, N, D, k, T, t_cur, t_next, tau, K_w, K_c, force, skip,
+                               m->idx, m->n_compute, target, m->cache_ws, m->cache_counters, m->cache_dec,
+                               m->err, s));
+    CS_TRY(record_end(m, 3, s, ev, 0.0));
+    CS_CUDA(cudaMemcpyAsync(m->n_host, m->n_compute, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
+    CS_CUDA(cudaMemcpyAsync(m->n_host + 1, m->err, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
+    CS_CUDA(cudaStreamSynchronize(s));
+    n_c = m->n_host[0];
+    if (m->n_host[1] != 0) {
+      cs::set_error("cs_search_step: device error %d recorded before step %d", m->n_host[1], k);
+      const int code = m->n_host[1];
+      cudaMemsetAsync(m->err, 0, sizeof(int), s);
+      return (cs_status)code;
+    }
   }
   if (n_out) *n_out = n_c;
-  CS_TRY(dit_forward_impl(m, x, m->idx, n_c, N, 1, t_cur, m->v, s));
+  CS_TRY(dit_forward_impl(m, x, idx, n_c, N, 1, t_cur, tokens ? nullptr : m->v, s));
   CS_TRY(record_begin(m, 3, s, ev));
-  if (n_c > 0 || target)
+  float* spart = static_cast<float*>(m->cache_ws) + (size_t)N * ((D + 8191) / 8192) * 2;
+  if (tokens) {
+    CS_TRY(cs::apply_tokens_run(x, x_ref, delta, accum, has_ref, skip, m->hout, idx, n_c, N, c.C, c.F, c.H, c.W,
+                                t_cur, t_next, target, scores, spart, m->tpart, N, m->err, s));
+  } else if (n_c > 0 || target) {
     CS_TRY(cs_cache_apply_computed(x, x_ref, delta, m->v, skip, N, D, t_cur, t_next, target, scores, m->cache_ws, s));
+  }
   // algorithmic bytes of indicator + update (each tensor read or written once):
-  //   skipped: read x, x_ref, Delta, write x                       16 D
-  //   computed: read x, v (+ x_ref on a free step), write x, Delta, x_ref   20 D (24 D)
+  //   skipped: read x, x_ref, Delta, write x                                 16 D
+  //   computed: read x, v (+ x_ref on a free step), write x, Delta, x_ref    20 D (24 D)
   const double skipped = N - n_c;
   double bytes = skipped * 16.0 * D + n_c * (wf ? 20.0 : 24.0) * D;
   if (target) bytes += 4.0 * D * N;

@@ -370,147 +370,174 @@ __global__ void score_finalize_kernel(const float* __restrict__ partials, int nc
   }
 }
 
-// ---------------------------------------------------- fused decide + skip ----
-// One cooperative launch per step: (1) drift partials of every (candidate, chunk) on a
-// free step, (2) a grid barrier, (3) every CTA derives all decisions from the partials
-// (the same fixed-order sums everywhere), CTA 0 stores the state and compaction list,
-// (4) skipped candidates get Eq. skip + Eq. euler (and their x0-score partials) while
-// computed ones wait for the DiT.  Phase (4) walks the chunks in reverse so the x just
-// read in phase (1) is still in L2.
+// ------------------------------------------------- single-pass decide + skip ----
+// Used by cs_search_step.  Two launches, no grid-wide barrier:
+//  drift_decide  every CTA takes a contiguous range of (candidate, chunk) items and
+//                writes their drift partials (x read with an L2 evict-last hint, so the
+//                skip update finds it in L2).  Per candidate, an arrival counter records
+//                how many of its chunks are done; the CTA that completes a candidate
+//                takes its decision (the same fixed-order sum of the same partials as
+//                the two-pass form, so the same bits), and the CTA that completes the
+//                last decision writes the compaction list.  Counters are left at zero.
+//  skip_update   launched with programmatic stream serialisation: its CTAs are
+//                scheduled while the first kernel drains and wait (griddepcontrol.wait)
+//                for its completion; each walks the same item range newest chunk first
+//                and applies Eq. skip + Eq. euler to skipped candidates.
+// No CTA ever waits for another CTA, so neither kernel needs co-resident CTAs.
 
-// Grid-wide barrier over co-resident CTAs (cooperative launch), bounded in time.
-// bar[0] counts arrivals, bar[1] is the generation; bar[0] must be 0 at launch.
-__device__ __forceinline__ void grid_barrier(unsigned* bar, int* err) {
-  block_sync();
-  if (threadIdx.x == 0) {
-    volatile unsigned* gen = bar + 1;
-    const unsigned g = *gen;
-    __threadfence();
-    if (atomicAdd(bar, 1u) == gridDim.x - 1) {
-      atomicExch(bar, 0u);
-      __threadfence();
-      atomicAdd(bar + 1, 1u);
-    } else {
-      const uint64_t t0 = globaltimer_ns();
-      while (*gen == g) {
-        __nanosleep(64);
-        if (globaltimer_ns() - t0 > CS_WAIT_TIMEOUT_NS) {
-          record_error(err, kErrTimeout);
-          break;
-        }
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait_primary() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// The decision of one candidate from its chunk partials (one warp; lane 0 writes).
+// Identical arithmetic to decide_finalize_kernel.  Returns 1 = compute (lane 0 only).
+__device__ __forceinline__ void decide_one(int i, const float* __restrict__ partials, int nch, bool free_step,
+                                           float a_before, bool had, float tau, const uint8_t* __restrict__ force,
+                                           float* __restrict__ accum, uint8_t* __restrict__ has_ref,
+                                           uint8_t* __restrict__ skip_mask, uint8_t* __restrict__ dec, int* err,
+                                           int lane) {
+  float num = 0.f, den = 0.f;
+  if (free_step) {
+    // partials written by other CTAs: read through L2 (never from this SM's L1)
+    float s0 = 0.f, s1 = 0.f;
+    for (int c = lane; c < nch; c += 32) {
+      s0 += __ldcg(partials + ((long long)i * nch + c) * 2 + 0);
+      s1 += __ldcg(partials + ((long long)i * nch + c) * 2 + 1);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      s0 += __shfl_xor_sync(0xffffffffu, s0, o);
+      s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+    }
+    num = s0;
+    den = s1;
+  }
+  if (lane == 0) {
+    bool compute = true;
+    float a = a_before;
+    if (free_step) {
+      const float drift = drift_of(num, den);
+      if (!isfinite(drift)) {
+        record_error(err, CS_ERR_NONFINITE);
+      } else {
+        a = a + drift;
+        compute = (tau <= 0.f) || (a > tau);
       }
     }
-    __threadfence();
+    if (force) {
+      const bool f = force[i] != 0;
+      if (!f && !had) {
+        record_error(err, CS_ERR_ARG);
+      } else {
+        compute = f;
+      }
+    }
+    accum[i] = compute ? 0.f : a;
+    skip_mask[i] = compute ? 0 : 1;
+    if (compute) has_ref[i] = 1;
+    dec[i] = compute ? 1 : 0;
   }
-  block_sync();
 }
 
-template <bool kScore>
-__global__ void __launch_bounds__(kCacheThreads) decide_skip_kernel(
-    float* __restrict__ x, const float* __restrict__ xr, const float* __restrict__ delta, float* __restrict__ accum,
-    uint8_t* __restrict__ has_ref, int N, long long D, int nch, int wf, float tau, const uint8_t* __restrict__ force,
-    uint8_t* __restrict__ skip_mask, int32_t* __restrict__ idx, int32_t* __restrict__ n_compute, float h,
-    float t_next, const float* __restrict__ target, float* __restrict__ partials, float* __restrict__ spart,
-    unsigned* bar, int* err) {
+__global__ void __launch_bounds__(kCacheThreads) drift_decide_kernel(
+    const float* __restrict__ x, const float* __restrict__ xr, float* __restrict__ accum,
+    uint8_t* __restrict__ has_ref, int N, long long D, int nch, float tau, const uint8_t* __restrict__ force,
+    uint8_t* __restrict__ skip_mask, uint8_t* __restrict__ dec, int32_t* __restrict__ idx,
+    int32_t* __restrict__ n_compute, float* __restrict__ partials, unsigned* __restrict__ counters, int* err) {
   __shared__ float red[2][32];
-  extern __shared__ float sm_dyn[];
-  float* a_s = sm_dyn;                                      // [N] accumulator before this step
-  uint8_t* had = reinterpret_cast<uint8_t*>(a_s + N);       // [N] has_ref before this step
-  uint8_t* dec = had + N;                                   // [N] 1 = compute, 0 = skip
+  __shared__ int s_flag, s_had;
+  __shared__ float s_a;
+  pdl_launch_dependents();   // the skip-update grid may be scheduled as soon as every CTA runs
   const int items = N * nch;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  // this CTA's contiguous range of (candidate, chunk) items
   const int per = (items + gridDim.x - 1) / gridDim.x;
   const int it0 = blockIdx.x * per, it1 = min(items, it0 + per);
-  // (0) snapshot the per-candidate state: CTA 0 rewrites it after the barrier
-  for (int i = threadIdx.x; i < N; i += blockDim.x) {
-    a_s[i] = accum[i];
-    had[i] = has_ref[i];
-  }
-  block_sync();
-  // (1) drift partials
-  if (!wf) {
-    for (int item = it0; item < it1; ++item) {
-      const int i = item / nch, c = item % nch;
-      if (!had[i]) continue;
-      const long long lo = (long long)c * kChunkElems, hi = min(D, lo + kChunkElems);
-      const float* xi = x + (long long)i * D + lo;
-      const float* ri = xr + (long long)i * D + lo;
-      const int n8 = (int)((hi - lo) >> 3);
-      float v[2] = {0.f, 0.f};
+  if (it0 >= it1) return;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int i_first = it0 / nch, i_last = (it1 - 1) / nch;
+  for (int i = i_first; i <= i_last; ++i) {
+    const int lo = max(it0, i * nch), hi = min(it1, (i + 1) * nch);
+    // the candidate's state before this step: read by one thread before this CTA's
+    // arrival (so before the deciding CTA can rewrite it) and shared with the others
+    if (threadIdx.x == 0) {
+      s_had = has_ref[i] != 0;
+      s_a = accum[i];
+    }
+    block_sync();
+    const bool had = s_had != 0;
+    const float a_before = s_a;
+    if (had) {
+      for (int item = lo; item < hi; ++item) {
+        const int c = item - i * nch;
+        const long long clo = (long long)c * kChunkElems, chi = min(D, clo + kChunkElems);
+        const float* xi = x + (long long)i * D + clo;
+        const float* ri = xr + (long long)i * D + clo;
+        const int n8 = (int)((chi - clo) >> 3);
+        float v[2] = {0.f, 0.f};
 #pragma unroll 4
-      for (int e = threadIdx.x; e < n8; e += kCacheThreads) {
-        const F8 a = ld8_keep(xi + 8 * e), b = ld8_once(ri + 8 * e);
+        for (int e = threadIdx.x; e < n8; e += kCacheThreads) {
+          const F8 a = ld8_keep(xi + 8 * e), b = ld8_once(ri + 8 * e);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const float dd = a.v[j] - b.v[j];
-          v[0] += dd * dd;
-          v[1] += b.v[j] * b.v[j];
+          for (int j = 0; j < 8; ++j) {
+            const float dd = a.v[j] - b.v[j];
+            v[0] += dd * dd;
+            v[1] += b.v[j] * b.v[j];
+          }
         }
-      }
-      block_sum<2>(v, red);
-      if (threadIdx.x == 0) {
-        partials[((long long)i * nch + c) * 2 + 0] = v[0];
-        partials[((long long)i * nch + c) * 2 + 1] = v[1];
-      }
-      block_sync();
-    }
-  }
-  // (2) every partial is written
-  grid_barrier(bar, err);
-  // (3) decisions (the same fixed-order sums in every CTA): CTA 0 takes every candidate
-  // and stores the state, the others only the candidates of their own range
-  const int c_lo = blockIdx.x == 0 ? 0 : (it0 < it1 ? it0 / nch : 0);
-  const int c_hi = blockIdx.x == 0 ? N : (it0 < it1 ? (it1 - 1) / nch + 1 : 0);
-  for (int i = c_lo + warp; i < c_hi; i += nw) {
-    const bool hr = had[i] != 0;
-    const bool free_step = !wf && hr;
-    float num = 0.f, den = 0.f;
-    if (free_step) {
-      num = warp_sum_partials_f32(partials + (long long)i * nch * 2 + 0, nch, 2, lane);
-      den = warp_sum_partials_f32(partials + (long long)i * nch * 2 + 1, nch, 2, lane);
-    }
-    if (lane == 0) {
-      bool compute = true;
-      float a = a_s[i];
-      if (free_step) {
-        const float drift = drift_of(num, den);
-        if (!isfinite(drift)) {
-          if (blockIdx.x == 0) record_error(err, CS_ERR_NONFINITE);
-        } else {
-          a = a + drift;
-          compute = (tau <= 0.f) || (a > tau);
+        block_sum<2>(v, red);
+        if (threadIdx.x == 0) {
+          partials[((long long)i * nch + c) * 2 + 0] = v[0];
+          partials[((long long)i * nch + c) * 2 + 1] = v[1];
         }
-      }
-      if (force) {
-        const bool f = force[i] != 0;
-        if (!f && !hr) {
-          if (blockIdx.x == 0) record_error(err, CS_ERR_ARG);
-        } else {
-          compute = f;
-        }
-      }
-      dec[i] = compute ? 1 : 0;
-      if (blockIdx.x == 0) {
-        accum[i] = compute ? 0.f : a;
-        skip_mask[i] = compute ? 0 : 1;
+        block_sync();
       }
     }
+    // arrival: this CTA's chunks of candidate i are done
+    if (threadIdx.x == 0) {
+      __threadfence();
+      const unsigned old = atomicAdd(&counters[i], (unsigned)(hi - lo));
+      s_flag = old + (unsigned)(hi - lo) == (unsigned)nch;
+    }
+    block_sync();
+    if (!s_flag) continue;
+    // this CTA completed candidate i: decide it
+    if (warp == 0) {
+      __threadfence();
+      decide_one(i, partials, nch, had, a_before, had, tau, force, accum, has_ref, skip_mask, dec, err, lane);
+      if (lane == 0) counters[i] = 0u;
+    }
+    block_sync();
+    if (threadIdx.x == 0) {
+      __threadfence();
+      s_flag = atomicAdd(&counters[N], 1u) == (unsigned)(N - 1);
+    }
+    block_sync();
+    if (s_flag && threadIdx.x == 0) {   // every candidate is decided: the compaction list
+      __threadfence();
+      const volatile uint8_t* dv = dec;
+      int n = 0;
+      for (int k = 0; k < N; ++k)
+        if (dv[k]) idx[n++] = k;
+      *n_compute = n;
+      counters[N] = 0u;
+    }
+    block_sync();
   }
-  block_sync();
-  if (blockIdx.x == 0 && threadIdx.x == 0) {
-    int n = 0;
-    for (int i = 0; i < N; ++i)
-      if (dec[i]) {
-        idx[n++] = i;
-        has_ref[i] = 1;
-      }
-    *n_compute = n;
-  }
-  // (4) skipped candidates of this range: x += h (x + Delta), newest chunks first
+}
+
+// Skipped candidates of the same item ranges: x += h (x + Delta), newest chunks first.
+template <bool kScore>
+__global__ void __launch_bounds__(kCacheThreads) skip_update_kernel(
+    float* __restrict__ x, const float* __restrict__ delta, const uint8_t* __restrict__ skip_mask, int N, long long D,
+    int nch, float h, float t_next, const float* __restrict__ target, float* __restrict__ spart) {
+  __shared__ float red[1][32];
+  pdl_wait_primary();        // the decisions (and every write of the first kernel) are visible
+  const int items = N * nch;
+  const int per = (items + gridDim.x - 1) / gridDim.x;
+  const int it0 = blockIdx.x * per, it1 = min(items, it0 + per);
   for (int item = it1 - 1; item >= it0; --item) {
     const int i = item / nch, c = item % nch;
-    if (dec[i]) continue;
+    if (!skip_mask[i]) continue;
     const long long lo = (long long)c * kChunkElems, hi = min(D, lo + kChunkElems);
     float* xi = x + (long long)i * D + lo;
     const float* di = delta + (long long)i * D + lo;
@@ -599,6 +626,86 @@ __global__ void __launch_bounds__(kCacheThreads) apply_computed_kernel(
   }
 }
 
+// ------------------------------------------------ computed update from tokens ----
+// The update of computed candidates straight from the DiT head's token-layout output, so
+// that the velocity never makes a round trip through HBM: the unpatchify scatter fused
+// with Eq. delta and Eq. euler.  For candidate i = idx[j] and latent element (c, f, h, w):
+//   v = hout[(j L + l) P + 4c + 2 (h & 1) + (w & 1)],  l = (f H/2 + h/2) W/2 + w/2,
+//   Delta = v - x,  x_ref = x,  x += (t_next - t_cur) v,  accum = 0, has_ref = 1, skip = 0.
+// One CTA per (token row (f, h/2), computed candidate): the row's W/2 tokens x P features
+// (contiguous in hout) are staged in shared memory as one float4 per (w/4, c, h&1) that
+// holds v at w..w+3, so hout and the four state tensors all move in 16-byte accesses.
+// The score partial of a tile is a fixed-order block sum (independent of the batch).
+template <bool kScore>
+__global__ void __launch_bounds__(kCacheThreads) velocity_update_kernel(
+    const float* __restrict__ hout, const int32_t* __restrict__ idx, int C, int F, int H, int W,
+    float* __restrict__ x, float* __restrict__ xr, float* __restrict__ delta, float* __restrict__ accum,
+    uint8_t* __restrict__ has_ref, uint8_t* __restrict__ skip_mask, float h, float t_next,
+    const float* __restrict__ target, float* __restrict__ tpart, long long idx_limit, int* err) {
+  extern __shared__ float4 s_v[];                 // [W/4][2C + 1]: the +1 staggers the banks
+  __shared__ float red[1][32];
+  const int H2 = H / 2, W2 = W / 2, W4 = W / 4, S = 2 * C + 1;
+  const int row = blockIdx.x, j = blockIdx.y;     // row = f * H/2 + h/2
+  const int f = row / H2, hh = row % H2;
+  const int i = idx[j];
+  if (!index_ok(i, idx_limit, err)) return;      // uniform over the CTA
+  const long long D = (long long)C * F * H * W;
+  const long long L = (long long)F * H2 * W2;
+  const float4* src = reinterpret_cast<const float4*>(hout + ((long long)j * L + (long long)row * W2) * (4 * C));
+  for (int q = threadIdx.x; q < W2 * C; q += kCacheThreads) {
+    const float4 a = __ldcs(src + q);             // features 4c..4c+3 of token T: (ph, pw) = 00 01 10 11
+    const int T = q / C, c = q % C;
+    float2* d = reinterpret_cast<float2*>(&s_v[(T >> 1) * S + 2 * c]) + (T & 1);
+    d[0] = make_float2(a.x, a.y);                 // h even: w = 2T, 2T + 1
+    d[2] = make_float2(a.z, a.w);                 // h odd
+  }
+  block_sync();
+  float* xi = x + (long long)i * D;
+  float* ri = xr + (long long)i * D;
+  float* di = delta + (long long)i * D;
+  float acc[1] = {0.f};
+  for (int q = threadIdx.x; q < 2 * C * W4; q += kCacheThreads) {
+    const int w4 = q % W4, cp = q / W4;           // cp = 2c + (h & 1)
+    const long long e = (((long long)(cp >> 1) * F + f) * H + 2 * hh + (cp & 1)) * W + 4 * w4;
+    const float4 vu = s_v[w4 * S + cp];
+    const float4 xv = __ldcs(reinterpret_cast<const float4*>(xi + e));
+    __stcs(reinterpret_cast<float4*>(di + e), make_float4(vu.x - xv.x, vu.y - xv.y, vu.z - xv.z, vu.w - xv.w));
+    __stcs(reinterpret_cast<float4*>(ri + e), xv);
+    const float4 xn = make_float4(xv.x + h * vu.x, xv.y + h * vu.y, xv.z + h * vu.z, xv.w + h * vu.w);
+    __stcs(reinterpret_cast<float4*>(xi + e), xn);
+    if (kScore) {
+      const float4 y = __ldg(reinterpret_cast<const float4*>(target + e));
+      const float e0 = xn.x - t_next * vu.x - y.x, e1 = xn.y - t_next * vu.y - y.y;
+      const float e2 = xn.z - t_next * vu.z - y.z, e3 = xn.w - t_next * vu.w - y.w;
+      acc[0] += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
+    }
+  }
+  if (kScore) {
+    block_sum<1>(acc, red);
+    if (threadIdx.x == 0) tpart[(long long)i * gridDim.x + row] = acc[0];
+  }
+  if (row == 0 && threadIdx.x == 0) {
+    accum[i] = 0.f;
+    has_ref[i] = 1;
+    skip_mask[i] = 0;
+  }
+}
+
+// Scores when the two kinds of candidates left their partials in different groupings:
+// skipped candidates per 8192-element chunk (nch), computed ones per token row (ntiles).
+__global__ void score_finalize_split_kernel(const float* __restrict__ spart, int nch, const float* __restrict__ tpart,
+                                            int ntiles, const uint8_t* __restrict__ skip_mask, int N,
+                                            float* __restrict__ scores) {
+  const int lane = threadIdx.x & 31;
+  const int w0 = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, nw = (gridDim.x * blockDim.x) >> 5;
+  for (int i = w0; i < N; i += nw) {
+    const bool sk = skip_mask[i] != 0;
+    const double s = sk ? warp_sum_partials(spart + (long long)i * nch, nch, 1, lane)
+                        : warp_sum_partials(tpart + (long long)i * ntiles, ntiles, 1, lane);
+    if (lane == 0) scores[i] = (float)(-sqrt(s));
+  }
+}
+
 // -------------------------------------------------------------------- top-k ----
 __global__ void topk_kernel(const float* __restrict__ scores, int N, int k, int32_t* __restrict__ idx) {
   extern __shared__ float s[];
@@ -649,9 +756,15 @@ __global__ void __launch_bounds__(kCacheThreads) beam_refill_kernel(
 
 using namespace cs;
 
+// Workspace layout: drift partials [N][nch][2], score partials [N][nch], then (at a
+// 256-byte boundary) the single-pass step's arrival counters [N + 1] and decisions [N].
+static size_t counters_offset(int N, long long D) {
+  return ((size_t)N * cache_chunks(D) * 3 * sizeof(float) + 255) / 256 * 256;
+}
+
 extern "C" size_t cs_cache_workspace_bytes(int N, long long D) {
   if (N <= 0 || D <= 0) return 0;
-  return (size_t)N * (size_t)cache_chunks(D) * 3 * sizeof(float) + 256;   // + grid-barrier words
+  return counters_offset(N, D) + (size_t)(N + 1) * sizeof(unsigned) + (size_t)N + 256;
 }
 
 extern "C" cs_status cs_cache_decide(const float* x, const float* x_ref, float* accum, uint8_t* has_ref, int N,
@@ -743,8 +856,101 @@ extern "C" cs_status cs_cache_apply_cfg(float* x, float* x_ref, float* delta, co
   return CS_OK;
 }
 
-// Bytes past cs_cache_workspace_bytes used by the fused pair: the grid-barrier words.
-static size_t barrier_offset(int N, long long D) { return (size_t)N * cache_chunks(D) * 3 * sizeof(float); }
+namespace cs {
+
+// The single-pass decide + skip of cs_search_step.  counters: N + 1 arrival counters, zero
+// on entry (every completed call leaves them at zero; the model keeps its own set, zeroed
+// when allocated, at a place that does not depend on N), and dec: N decision bytes; both
+// nullptr: the set inside the workspace, whose counters are cleared first.
+cs_status decide_skip_run(float* x, const float* x_ref, const float* delta, float* accum, uint8_t* has_ref, int N,
+                          long long D, int step_k, int T, float t_cur, float t_next, float tau, int K_w, int K_c,
+                          const uint8_t* force, uint8_t* skip_mask, int32_t* idx, int32_t* n_compute,
+                          const float* target, void* workspace, unsigned* counters, uint8_t* dec, int* err,
+                          cudaStream_t stream) {
+  const int nch = cache_chunks(D);
+  const int wf = window_forced(step_k, T, K_w, K_c) ? 1 : 0;
+  if (wf && !force) {
+    decide_all_compute_kernel<<<1, 256, 0, stream>>>(accum, has_ref, N, skip_mask, idx, n_compute);
+    CS_LAUNCHED();
+    return CS_OK;
+  }
+  float* partials = static_cast<float*>(workspace);
+  float* spart = partials + (size_t)N * nch * 2;
+  const bool counters_zero = counters != nullptr;
+  if (!counters) {
+    counters = reinterpret_cast<unsigned*>(static_cast<char*>(workspace) + counters_offset(N, D));
+    dec = reinterpret_cast<uint8_t*>(counters + N + 1);
+  }
+  const int items = N * nch;
+  int grid = num_sms() * 4;   // 4 CTAs of 256 threads per SM keep enough 32-byte loads in flight
+  if (grid > items) grid = items;
+  if (wf) {
+    // forced mask inside the window: no drift is evaluated, one CTA decides
+    decide_finalize_kernel<<<1, 1024, N, stream>>>(partials, nch, accum, has_ref, N, 1, tau, force, skip_mask, idx,
+                                                  n_compute, err);
+    CS_LAUNCHED();
+  } else {
+    if (!counters_zero) CS_CUDA(cudaMemsetAsync(counters, 0, (size_t)(N + 1) * sizeof(unsigned), stream));
+    drift_decide_kernel<<<grid, kCacheThreads, 0, stream>>>(x, x_ref, accum, has_ref, N, D, nch, tau, force,
+                                                           skip_mask, dec, idx, n_compute, partials, counters, err);
+    CS_LAUNCHED();
+  }
+  const float h = t_next - t_cur;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kCacheThreads);
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (target)
+    CS_CUDA(cudaLaunchKernelEx(&cfg, skip_update_kernel<true>, x, delta, (const uint8_t*)skip_mask, N, D, nch, h,
+                               t_next, target, spart));
+  else
+    CS_CUDA(cudaLaunchKernelEx(&cfg, skip_update_kernel<false>, x, delta, (const uint8_t*)skip_mask, N, D, nch, h,
+                               t_next, (const float*)nullptr, (float*)nullptr));
+  CS_LAUNCHED();
+  return CS_OK;
+}
+
+cs_status apply_tokens_run(float* x, float* x_ref, float* delta, float* accum, uint8_t* has_ref, uint8_t* skip_mask,
+                           const float* hout, const int32_t* idx, int n_c, int N, int C, int F, int H, int W,
+                           float t_cur, float t_next, const float* target, float* scores, const float* spart,
+                           float* tpart, long long idx_limit, int* err, cudaStream_t stream) {
+  const long long D = (long long)C * F * H * W;
+  const int ntiles = F * (H / 2);
+  const float h = t_next - t_cur;
+  const size_t smem = (size_t)(W / 4) * (2 * C + 1) * sizeof(float4);
+  if (n_c > 0) {
+    const dim3 grid(ntiles, n_c);
+    if (target)
+      velocity_update_kernel<true><<<grid, kCacheThreads, smem, stream>>>(hout, idx, C, F, H, W, x, x_ref, delta,
+                                                                         accum, has_ref, skip_mask, h, t_next, target,
+                                                                         tpart, idx_limit, err);
+    else
+      velocity_update_kernel<false><<<grid, kCacheThreads, smem, stream>>>(hout, idx, C, F, H, W, x, x_ref, delta,
+                                                                          accum, has_ref, skip_mask, h, t_next,
+                                                                          nullptr, nullptr, idx_limit, err);
+    CS_LAUNCHED();
+  }
+  if (target) {
+    score_finalize_split_kernel<<<(N + 3) / 4, 128, 0, stream>>>(spart, cache_chunks(D), tpart, ntiles, skip_mask, N,
+                                                                 scores);
+    CS_LAUNCHED();
+  }
+  return CS_OK;
+}
+
+// Whether apply_tokens_run handles this latent shape (16-byte rows along W and a staging
+// tile that fits the default shared memory of a CTA).
+bool apply_tokens_supported(int C, int F, int H, int W) {
+  return C > 0 && F > 0 && H > 0 && W > 0 && (H % 2) == 0 && (W % 4) == 0 &&
+         (size_t)(W / 4) * (2 * C + 1) * sizeof(float4) <= 48 * 1024;
+}
+
+}  // namespace cs
 
 extern "C" cs_status cs_cache_decide_skip(float* x, const float* x_ref, const float* delta, float* accum,
                                           uint8_t* has_ref, int N, long long D, int step_k, int T, float t_cur,
@@ -759,38 +965,29 @@ extern "C" cs_status cs_cache_decide_skip(float* x, const float* x_ref, const fl
                  (reinterpret_cast<uintptr_t>(x_ref) & 31) == 0 && (reinterpret_cast<uintptr_t>(delta) & 31) == 0 &&
                  (!target || (reinterpret_cast<uintptr_t>(target) & 31) == 0),
              "cs_cache_decide_skip: needs D %% 8 == 0 and 32-byte aligned tensors");
-  const int nch = cache_chunks(D);
-  int wf = window_forced(step_k, T, K_w, K_c) ? 1 : 0;
-  if (wf && !force) {
-    decide_all_compute_kernel<<<1, 256, 0, stream>>>(accum, has_ref, N, skip_mask, idx, n_compute);
-    CS_LAUNCHED();
-    return CS_OK;
-  }
-  float* partials = static_cast<float*>(workspace);
-  float* spart = partials + (size_t)N * nch * 2;
-  unsigned* bar = reinterpret_cast<unsigned*>(static_cast<char*>(workspace) + barrier_offset(N, D));
-  CS_CUDA(cudaMemsetAsync(bar, 0, 2 * sizeof(unsigned), stream));
-  float h = t_next - t_cur;
-  const bool score = target != nullptr;
-  void* kern = score ? (void*)decide_skip_kernel<true> : (void*)decide_skip_kernel<false>;
-  int per_sm = 0;
-  const size_t dyn = (size_t)N * 6;
-  CS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kCacheThreads, dyn));
-  if (per_sm < 1) {
-    set_error("cs_cache_decide_skip: kernel does not fit on an SM");
-    return CS_ERR_CUDA;
-  }
-  // at most 4 CTAs per SM: a smaller cooperative grid launches and crosses the barrier
-  // faster, and 4 x 256 threads still keep enough loads in flight (measured on GB300)
-  int grid = num_sms() * (per_sm < 4 ? per_sm : 4);
-  const int items = N * nch;
-  if (grid > items) grid = items;
-  void* args[] = {&x, (void*)&x_ref, (void*)&delta, &accum, &has_ref, &N, &D, (void*)&nch, &wf, &tau,
-                  (void*)&force, &skip_mask, &idx, &n_compute, &h, &t_next, (void*)&target, &partials, &spart, &bar,
-                  &err};
-  CS_CUDA(cudaLaunchCooperativeKernel(kern, dim3(grid), dim3(kCacheThreads), args, dyn, stream));
-  count_launch();
-  return CS_OK;
+  return decide_skip_run(x, x_ref, delta, accum, has_ref, N, D, step_k, T, t_cur, t_next, tau, K_w, K_c, force,
+                         skip_mask, idx, n_compute, target, workspace, nullptr, nullptr, err, stream);
+}
+
+extern "C" cs_status cs_cache_apply_tokens(float* x, float* x_ref, float* delta, float* accum, uint8_t* has_ref,
+                                           uint8_t* skip_mask, const float* hout, const int32_t* idx, int n_c, int N,
+                                           int C, int F, int H, int W, float t_cur, float t_next,
+                                           const float* target, float* scores, void* workspace, float* tile_partials,
+                                           int* err, cudaStream_t stream) {
+  CS_REQUIRE(N > 0 && N <= 4096 && n_c >= 0 && n_c <= N, "cs_cache_apply_tokens: need 0 <= n_c <= N <= 4096");
+  CS_REQUIRE(x && x_ref && delta && accum && has_ref && skip_mask && (n_c == 0 || (hout && idx)),
+             "cs_cache_apply_tokens: null pointer");
+  CS_REQUIRE(apply_tokens_supported(C, F, H, W), "cs_cache_apply_tokens: needs even H and W %% 4 == 0 (W=%d)", W);
+  CS_REQUIRE(!target || (scores && workspace && tile_partials),
+             "cs_cache_apply_tokens: scoring needs scores, workspace and tile_partials");
+  const uintptr_t al = reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(x_ref) |
+                       reinterpret_cast<uintptr_t>(delta) | reinterpret_cast<uintptr_t>(hout) |
+                       reinterpret_cast<uintptr_t>(target);
+  CS_REQUIRE((al & 15) == 0, "cs_cache_apply_tokens: tensors must be 16-byte aligned");
+  const long long D = (long long)C * F * H * W;
+  const float* spart = workspace ? static_cast<const float*>(workspace) + (size_t)N * cache_chunks(D) * 2 : nullptr;
+  return apply_tokens_run(x, x_ref, delta, accum, has_ref, skip_mask, hout, idx, n_c, N, C, F, H, W, t_cur, t_next,
+                          target, scores, spart, tile_partials, (long long)N, err, stream);
 }
 
 extern "C" cs_status cs_cache_apply_computed(float* x, float* x_ref, float* delta, const float* v,

@@ -59,7 +59,7 @@ def main():
     build.build()
     from paper_2607_23159_gb300 import binding as B
     ap = argparse.ArgumentParser()
-    ap.add_argument("kernel", choices=["attention", "gemm", "qkv", "layernorm", "cache", "cache-fused"])
+    ap.add_argument("kernel", choices=["attention", "gemm", "qkv", "layernorm", "cache", "cache-fused", "cache-tokens"])
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--L", type=int, default=32760)
     ap.add_argument("--Lk", type=int, default=None)
@@ -71,6 +71,7 @@ def main():
     ap.add_argument("--epi", type=int, default=1)
     ap.add_argument("--D", type=int, default=2096640)
     ap.add_argument("--skip-frac", type=float, default=1.0)
+    ap.add_argument("--latent", default="16x21x60x104", help="C x F x H x W of the latent (cache-tokens)")
     ap.add_argument("--reps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=2)
     ap.add_argument("--torch", action="store_true", help="time the PyTorch comparator instead")
@@ -155,6 +156,9 @@ def main():
         out.update(shape=dict(M=M, d=d), ms=ms, gbs=M * d * 6.0 / (ms / 1e3) / 1e9)
     else:
         N, D = a.N, a.D
+        lat = [int(v) for v in a.latent.split("x")]
+        if a.kernel == "cache-tokens":
+            D = lat[0] * lat[1] * lat[2] * lat[3]
         st = B.new_state(N, D)
         st["x"].normal_()
         st["x_ref"].copy_(st["x"] * 0.99)
@@ -166,9 +170,17 @@ def main():
         idx = torch.zeros(N, dtype=torch.int32, device=dev)
         nc = torch.zeros(1, dtype=torch.int32, device=dev)
         force = (torch.rand(N, device=dev) >= a.skip_frac).to(torch.uint8)
+        n_comp = int(force.sum())
+        C_, F_, H_, W_ = lat
+        hout = torch.randn(max(1, n_comp) * F_ * (H_ // 2) * (W_ // 2), 4 * C_, device=dev)
+        comp_idx = torch.nonzero(force).to(torch.int32).reshape(-1)
 
         def run():
-            if a.kernel == "cache-fused":
+            if a.kernel == "cache-tokens":   # the search step's pair: decide + skip, then the computed update
+                B.cache_decide_skip(st["x"], st["x_ref"], st["delta"], st["accum"], st["has_ref"], 20, 50, 0.6, 0.58,
+                                    0.1, 5, 5, skip, idx, nc, ws, force=force)
+                B.cache_apply_tokens(st, skip, hout, comp_idx, n_comp, C_, F_, H_, W_, 0.6, 0.58)
+            elif a.kernel == "cache-fused":
                 B.cache_decide_skip(st["x"], st["x_ref"], st["delta"], st["accum"], st["has_ref"], 20, 50, 0.6, 0.58,
                                     0.1, 5, 5, skip, idx, nc, ws, force=force)
                 B.cache_apply_computed(st["x"], st["x_ref"], st["delta"], v, skip, 0.6, 0.58)

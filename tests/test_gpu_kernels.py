@@ -356,3 +356,70 @@ def test_fused_decide_skip_equals_two_pass_path(B, N, D, score):
     assert 0 < int(out[0][1][0].sum()) < N or 0 < int(out[0][2][0].sum()) < N   # some candidates skip
     for key in ("x", "x_ref", "delta", "accum", "has_ref"):
         assert torch.equal(states[0][key], states[1][key]), key
+
+
+@pytest.mark.parametrize("m,k,score", [(synth.WAN_1_3B, 20, True), (synth.WAN_1_3B, 21, False),
+                                        (synth.TINY, 5, True), (synth.WAN_1_3B_SHORT, 3, True)])
+def test_apply_tokens_equals_scatter_then_apply(B, m, k, score):
+    """cs_cache_apply_tokens (the computed update straight from the head's token-layout
+    output) gives the state bits of the velocity scatter (the oracle's unpatchify) followed
+    by cs_cache_apply_computed; skipped candidates are left alone; scores agree.  Step 3
+    of the short workload lies in its warm-up window: every candidate computes."""
+    N, T, tau = 4, 50 if m is not synth.TINY else 10, 0.1
+    K = 5 if T == 50 else 3
+    D, L = m.D, m.L
+    t = O.time_grid(T)
+    x = synth.normal(61, (N, D))
+    xr = x + synth.normal(62, (N, D)) * np.array([0.02, 0.2, 0.01, 0.3])[:, None]
+    states = []
+    for _ in range(2):
+        st = B.new_state(N, D)
+        st["x"].copy_(dev(x))
+        st["x_ref"].copy_(dev(xr))
+        st["delta"].copy_(dev(synth.normal(63, (N, D))))
+        st["accum"].copy_(dev(np.array([0.01, 0.0, 0.02, 0.0], np.float32)))
+        st["has_ref"].fill_(1)
+        states.append(st)
+    y = dev(synth.normal(64, (D,)))
+    hout_all = synth.normal(65, (N * L, 4 * m.C))
+    out = []
+    for which, st in enumerate(states):
+        ws = torch.zeros(B.cache_workspace_bytes(N, D) // 4 + 1, device="cuda")
+        skip = torch.zeros(N, dtype=torch.uint8, device="cuda")
+        idx = torch.zeros(N, dtype=torch.int32, device="cuda")
+        nc = torch.zeros(1, dtype=torch.int32, device="cuda")
+        sc = torch.zeros(N, device="cuda")
+        err = err_word()
+        tgt = y if score else None
+        B.cache_decide_skip(st["x"], st["x_ref"], st["delta"], st["accum"], st["has_ref"], k, T, float(t[k - 1]),
+                            float(t[k]), tau, K, K, skip, idx, nc, ws, target=tgt, err=err)
+        torch.cuda.synchronize()
+        n_c = int(nc[0])
+        comp = idx[:n_c].cpu().numpy()
+        hout = dev(hout_all[:n_c * L])
+        if which == 0:
+            v = torch.full((N, D), float("nan"), device="cuda")
+            for j, i in enumerate(comp):
+                v[i] = dev(O.unpatchify(hout_all[j * L:(j + 1) * L], m.C, m.F, m.H, m.W).reshape(-1))
+            B.cache_apply_computed(st["x"], st["x_ref"], st["delta"], v, skip, float(t[k - 1]), float(t[k]),
+                                   workspace=ws, target=tgt, scores=sc if score else None)
+        else:
+            tp = torch.zeros(N, m.F * m.H // 2, device="cuda")
+            B.cache_apply_tokens(st, skip, hout, idx, n_c, m.C, m.F, m.H, m.W, float(t[k - 1]), float(t[k]),
+                                 workspace=ws, target=tgt, scores=sc if score else None, tile_partials=tp, err=err)
+        torch.cuda.synchronize()
+        assert int(err[0]) == 0
+        out.append((skip.cpu(), comp, sc.cpu()))
+    (s0, c0, sc0), (s1, c1, sc1) = out
+    assert torch.equal(s0, s1) and np.array_equal(c0, c1)
+    if k > K and k <= T - K:
+        assert s0.tolist() == [1, 0, 1, 0]           # drifts 0.02, 0.2, 0.01, 0.3 against tau 0.1
+    else:
+        assert not s0.any()
+    for key in ("x", "x_ref", "delta", "accum", "has_ref"):
+        assert torch.equal(states[0][key], states[1][key]), key
+    if score:
+        torch.testing.assert_close(sc0, sc1, rtol=1e-6, atol=0)
+        ref = [O.score(states[0]["x"][i].double().cpu().numpy() - t[k] * (
+            states[0]["x"][i].double().cpu().numpy() - x[i]) / (t[k] - t[k - 1]), y.cpu().numpy()) for i in range(N)]
+        np.testing.assert_allclose(sc1.numpy(), ref, rtol=1e-4)

@@ -339,3 +339,23 @@ def test_kernel_stats_count_the_algorithmic_work(B, tiny):
     assert stats[B.KC_CACHE][2] == float(m.D * N * (20 * (T - free) + 24 * free))
     for c in range(5):
         assert stats[c][0] > 0 and stats[c][1] > 0.0, c
+
+
+def test_searches_of_changing_sizes_on_one_model(B):
+    """The single-pass cache step keeps its per-candidate arrival counters in the model
+    between steps; a model that has run searches of other sizes (larger and smaller)
+    gives each search the same bits as a fresh model."""
+    inp = Inputs(synth.TINY, 8)
+    shared = _model(B, inp, 8)
+    for N in (4, 6, 2, 8, 3):
+        sub = Inputs.__new__(Inputs)
+        sub.__dict__.update(inp.__dict__)
+        sub.x1 = inp.x1[:N]
+        s1, m1, sc1, n1 = gpu_search(B, sub, N, 10, 0.1, 1, 1, model=shared)
+        fresh = _model(B, inp, 8)
+        s2, m2, sc2, n2 = gpu_search(B, sub, N, 10, 0.1, 1, 1, model=fresh)
+        fresh.close()
+        assert n1 == n2 and np.array_equal(m1, m2), N
+        assert torch.equal(s1["x"], s2["x"]) and np.array_equal(sc1, sc2), N
+        assert 0 < m1.sum() < m1.size, N        # both kinds of decision occur
+    shared.close()
