@@ -18,6 +18,7 @@ from __future__ import annotations
 
 import argparse
 import functools
+import hashlib
 import json
 import os
 import statistics
@@ -31,10 +32,34 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "candidate-denoising-steps/sec at Wan2.1-1.3B shape"
-# DRAM bytes (read + write) of one self-attention launch per (candidate, head) at 32760
-# tokens, hd 128, from the ncu capture in profiles/attn_tcgen05_hd128_L32760.md
-ATTN_DRAM_BYTES_PER_HEAD_L32760 = 384.8e6 / 12
 UNIT = "candidate-steps/s"
+COUNTERS = os.path.join(ROOT, "profiles", "kernel_counters.txt")
+
+
+def kernel_counters(cls, path=COUNTERS):
+    """The committed ncu counters of kernel class ``cls`` (one ``key=value`` line per
+    capture), with ``stale`` set when the kernel's source file has changed since the
+    capture (its SHA-256 prefix differs).  None when there is no capture of the class."""
+    try:
+        lines = open(path).read().splitlines()
+    except OSError:
+        return None
+    for line in lines:
+        if line.startswith("#") or not line.strip():
+            continue
+        rec = dict(f.split("=", 1) for f in line.split() if "=" in f)
+        if rec.get("class") != cls:
+            continue
+        src, sha = rec["src"].split(":")
+        try:
+            cur = hashlib.sha256(open(os.path.join(ROOT, "paper_2607_23159_gb300", "csrc", src), "rb").read())
+            rec["stale"] = cur.hexdigest()[:16] != sha
+        except OSError:
+            rec["stale"] = True
+        for k in ("units", "dram_bytes", "tensor_active", "sm_mhz"):
+            rec[k] = float(rec[k])
+        return rec
+    return None
 
 
 def parse():
@@ -399,7 +424,15 @@ def run_ours(args, cfg):
     peak_tf = peak_tf or 1700.0
     ach = (fl_sa / n_sa) / (ms_sa / n_sa / 1e3) / 1e12 if n_sa else 0.0
     heads_per_launch = (fl_sa / n_sa) / (4.0 * m.L * m.L * m.hd) if n_sa else 0.0
-    traffic = heads_per_launch * ATTN_DRAM_BYTES_PER_HEAD_L32760 if (m.L == 32760 and m.hd == 128) else None
+    clocks = clk.summary()
+    # the measured peak was taken at the clock MEASURED_PEAKS records under load; scaled to
+    # this run's median SM clock it is the peak the kernel could reach here
+    peak_mhz = (peaks.get("clocks_under_load") or {}).get("sm_mhz_median")
+    matched = (ach / (peak_tf * clocks["sm_mhz"] / peak_mhz)) if (peak_mhz and clocks.get("sm_mhz")) else None
+    ctr_sa = kernel_counters("self_attention")
+    fresh_sa = ctr_sa is not None and not ctr_sa["stale"] and m.L == 32760 and m.hd == 128
+    traffic = heads_per_launch * ctr_sa["dram_bytes"] / ctr_sa["units"] if fresh_sa else None
+    ctr_g = kernel_counters("gemm")
     n_g, ms_g, fl_g = stats[B.KC_GEMM]
     n_c, ms_c, by_c = stats[B.KC_CACHE]
     hbm = peaks.get("hbm_gbs") or 6800.0
@@ -411,10 +444,20 @@ def run_ours(args, cfg):
         "config": workload_config(args, cfg),
         "roofline": {"kernel": "self-attention (tcgen05 flash attention)", "bound": "tensor", "achieved": ach,
                      "peak": peak_tf, "peak_source": peak_src, "unit": "TFLOP/s", "frac": ach / peak_tf,
-                     "traffic": traffic, "launches": n_sa, "avg_ms": ms_sa / n_sa if n_sa else None},
+                     "traffic": traffic, "launches": n_sa, "avg_ms": ms_sa / n_sa if n_sa else None,
+                     "sm_mhz": clocks["sm_mhz"], "peak_sm_mhz": peak_mhz, "frac_clock_matched": matched,
+                     "tensor_pipe_active_ncu": (ctr_sa["tensor_active"] / 100.0) if fresh_sa else None,
+                     "ncu_sm_mhz": ctr_sa["sm_mhz"] if fresh_sa else None,
+                     "ncu_counters": ("stale: kernel source changed since the capture" if ctr_sa and ctr_sa["stale"]
+                                      else (ctr_sa["summary"] if ctr_sa else None))},
         "kernels": {
             "gemm": {"launches": n_g, "ms": ms_g, "tflops": fl_g / (ms_g / 1e3) / 1e12 if ms_g else None,
-                     "frac": (fl_g / (ms_g / 1e3) / 1e12) / peak_tf if ms_g else None},
+                     "frac": (fl_g / (ms_g / 1e3) / 1e12) / peak_tf if ms_g else None,
+                     "frac_clock_matched": ((fl_g / (ms_g / 1e3) / 1e12) / (peak_tf * clocks["sm_mhz"] / peak_mhz)
+                                            if (ms_g and peak_mhz and clocks.get("sm_mhz")) else None),
+                     "tensor_pipe_active_ncu": (ctr_g["tensor_active"] / 100.0
+                                                if ctr_g and not ctr_g["stale"] else None),
+                     "ncu_kernel": ctr_g["kernel"] if ctr_g else None},
             "self_attention": {"launches": n_sa, "ms": ms_sa},
             "cross_attention": {"launches": stats[B.KC_CROSS_ATTN][0], "ms": stats[B.KC_CROSS_ATTN][1]},
             "cache_update": {"launches": n_c, "ms": ms_c, "gbs": cache_gbs, "frac_hbm": cache_gbs / hbm},
@@ -422,7 +465,7 @@ def run_ours(args, cfg):
         },
         "computed_fraction": computed / ((2 if mode == "cfg" else 1) * advanced),
         "gpu_launches": launches,
-        "clocks": clk.summary(),
+        "clocks": clocks,
     }
     if e2e:
         line["e2e"] = e2e

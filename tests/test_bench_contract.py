@@ -46,3 +46,20 @@ def test_clock_summary_parses_nvidia_smi_samples():
     empty = bench.ClockSampler(0)
     empty.out = ""
     assert empty.summary()["reasons"] == ["unsampled"]
+
+
+def test_committed_kernel_counters_parse_and_track_their_source(tmp_path):
+    """The roofline's ncu evidence comes from profiles/kernel_counters.txt: every capture
+    line names its class, units, DRAM bytes and tensor-pipe activity, and a capture whose
+    kernel source hash no longer matches is reported as stale (its figures are dropped)."""
+    sys.path.insert(0, ROOT)
+    import bench
+    rec = bench.kernel_counters("self_attention")
+    assert rec is not None and rec["units"] > 0 and rec["dram_bytes"] > 0 and 0 < rec["tensor_active"] <= 100
+    assert os.path.exists(os.path.join(ROOT, "profiles", rec["summary"]))
+    fake = tmp_path / "c.txt"
+    fake.write_text("# comment\nclass=self_attention kernel=k units=2 dram_bytes=1e6 tensor_active=50 sm_mhz=1900 "
+                    "src=attention.cu:0000000000000000 summary=x.md\n")
+    old = bench.kernel_counters("self_attention", path=str(fake))
+    assert old["stale"] is True and old["units"] == 2.0
+    assert bench.kernel_counters("no_such_class", path=str(fake)) is None
