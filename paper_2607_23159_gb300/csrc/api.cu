@@ -55,8 +55,8 @@ struct cs_model {
   float *resid, *hout, *cond_scratch, *mods, *hmod, *v, *x_host_stage;
   int32_t *idx, *n_compute;
   int32_t* idx_all;   // 0, 1, ..., max_batch - 1: the compaction list of an all-compute step
-  unsigned* cache_counters;   // arrival counters [max_batch + 1] (zero between steps)
-  uint8_t* cache_dec;         // decisions [max_batch]
+  unsigned* cache_counter;    // arrival counter of the decision pass (zero between steps)
+  int32_t* cache_sidx;        // skipped candidates [max_batch] and their count
   float* tpart;       // score partials of computed candidates per token row [max_batch][F*H/2]
   bool tokens_update = false;   // computed update straight from the head's token output
   uint8_t* skip_tmp;
@@ -84,6 +84,15 @@ cs_status record_end(cs_model* m, int cls, cudaStream_t s, cudaEvent_t* ev, doub
   CS_CUDA(cudaEventRecord(ev[1], s));
   m->timing[cls].pending.emplace_back(ev[0], ev[1]);
   m->timing[cls].pending_work.push_back(work);
+  return CS_OK;
+}
+
+// Work of a class that launched nothing more: added to its last timed region.
+cs_status add_work(cs_model* m, int cls, double work) {
+  if (!m->profiling) return CS_OK;
+  Timing& t = m->timing[cls];
+  if (!t.pending_work.empty()) t.pending_work.back() += work;
+  else t.work += work;
   return CS_OK;
 }
 
@@ -252,8 +261,8 @@ extern "C" cs_status cs_init_model(const cs_model_config* cfg, cs_model** out) {
   addf(&m->x_host_stage, (size_t)cfg->max_batch * m->D);
   items.push_back({reinterpret_cast<void**>(&m->idx), (size_t)cfg->max_batch * 4});
   items.push_back({reinterpret_cast<void**>(&m->idx_all), (size_t)cfg->max_batch * 4});
-  items.push_back({reinterpret_cast<void**>(&m->cache_counters), (size_t)(cfg->max_batch + 1) * 4});
-  items.push_back({reinterpret_cast<void**>(&m->cache_dec), (size_t)cfg->max_batch});
+  items.push_back({reinterpret_cast<void**>(&m->cache_counter), 4});
+  items.push_back({reinterpret_cast<void**>(&m->cache_sidx), (size_t)(cfg->max_batch + 1) * 4});
   addf(&m->tpart, (size_t)cfg->max_batch * cfg->F * (cfg->H / 2));
   items.push_back({reinterpret_cast<void**>(&m->n_compute), 16});
   items.push_back({reinterpret_cast<void**>(&m->skip_tmp), (size_t)cfg->max_batch});
@@ -280,6 +289,12 @@ extern "C" cs_status cs_init_model(const cs_model_config* cfg, cs_model** out) {
   for (int i = 0; i < cfg->max_batch; ++i) iota[i] = i;
   cudaMemcpy(m->idx_all, iota.data(), iota.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
   m->tokens_update = cs::apply_tokens_supported(cfg->C, cfg->F, cfg->H, cfg->W);
+  if (cs::load_cache_kernels() != CS_OK) {
+    cudaFree(m->ws);
+    cudaFree(m->wmem);
+    delete m;
+    return CS_ERR_CUDA;
+  }
   std::vector<float*> offs(nb);
   for (size_t b = 0; b < nb; ++b) offs[b] = m->blk[b].mod_off;
   cudaMemcpy(m->mod_offs_dev, offs.data(), nb * sizeof(float*), cudaMemcpyHostToDevice);
@@ -547,8 +562,8 @@ static cs_status step_impl(cs_model* m, float* x, float* x_ref, float* delta, fl
     // decisions + the update of skipped candidates; computed ones after the DiT
     CS_TRY(record_begin(m, 3, s, ev));
     CS_TRY(cs::decide_skip_run(x, x_ref, delta, accum, has_ref, N, D, k, T, t_cur, t_next, tau, K_w, K_c, force, skip,
-                               m->idx, m->n_compute, target, m->cache_ws, m->cache_counters, m->cache_dec,
-                               m->err, s));
+                               m->idx, m->n_compute, target, m->cache_ws,
+                               cs::StepScratch{m->cache_counter, m->cache_sidx}, m->err, s));
     CS_TRY(record_end(m, 3, s, ev, 0.0));
     CS_CUDA(cudaMemcpyAsync(m->n_host, m->n_compute, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
     CS_CUDA(cudaMemcpyAsync(m->n_host + 1, m->err, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
@@ -563,6 +578,13 @@ static cs_status step_impl(cs_model* m, float* x, float* x_ref, float* delta, fl
   }
   if (n_out) *n_out = n_c;
   CS_TRY(dit_forward_impl(m, x, idx, n_c, N, 1, t_cur, tokens ? nullptr : m->v, s));
+  // algorithmic bytes of indicator + update (each tensor read or written once):
+  //   skipped: read x, x_ref, Delta, write x                                 16 D
+  //   computed: read x, v (+ x_ref on a free step), write x, Delta, x_ref    20 D (24 D)
+  const double skipped = N - n_c;
+  double bytes = skipped * 16.0 * D + n_c * (wf ? 20.0 : 24.0) * D;
+  if (target) bytes += 4.0 * D * N;
+  if (n_c == 0 && !target) return add_work(m, 3, bytes);   // the decision pass did the whole update
   CS_TRY(record_begin(m, 3, s, ev));
   float* spart = static_cast<float*>(m->cache_ws) + (size_t)N * ((D + 8191) / 8192) * 2;
   if (tokens) {
@@ -571,12 +593,6 @@ static cs_status step_impl(cs_model* m, float* x, float* x_ref, float* delta, fl
   } else if (n_c > 0 || target) {
     CS_TRY(cs_cache_apply_computed(x, x_ref, delta, m->v, skip, N, D, t_cur, t_next, target, scores, m->cache_ws, s));
   }
-  // algorithmic bytes of indicator + update (each tensor read or written once):
-  //   skipped: read x, x_ref, Delta, write x                                 16 D
-  //   computed: read x, v (+ x_ref on a free step), write x, Delta, x_ref    20 D (24 D)
-  const double skipped = N - n_c;
-  double bytes = skipped * 16.0 * D + n_c * (wf ? 20.0 : 24.0) * D;
-  if (target) bytes += 4.0 * D * N;
   CS_TRY(record_end(m, 3, s, ev, bytes));
   return CS_OK;
 }

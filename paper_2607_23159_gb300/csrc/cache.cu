@@ -16,6 +16,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "elementwise.h"
 #include "ptx.cuh"
 
 namespace cs {
@@ -156,7 +157,8 @@ __device__ __forceinline__ float drift_of(float num, float den) { return sqrtf(n
 __global__ void decide_finalize_kernel(const float* __restrict__ partials, int nch, float* __restrict__ accum,
                                        uint8_t* __restrict__ has_ref, int N, int window_forced_step, float tau,
                                        const uint8_t* __restrict__ force, uint8_t* __restrict__ skip_mask,
-                                       int32_t* __restrict__ idx, int32_t* __restrict__ n_compute, int* err) {
+                                       int32_t* __restrict__ idx, int32_t* __restrict__ n_compute, int* err,
+                                       int32_t* __restrict__ sidx = nullptr) {
   extern __shared__ uint8_t flags[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
   for (int i = warp; i < N; i += nw) {
@@ -201,10 +203,13 @@ __global__ void decide_finalize_kernel(const float* __restrict__ partials, int n
   }
   block_sync();
   if (threadIdx.x == 0) {
-    int n = 0;
-    for (int i = 0; i < N; ++i)
+    int n = 0, ns = 0;
+    for (int i = 0; i < N; ++i) {
       if (flags[i]) idx[n++] = i;
+      else if (sidx) sidx[ns++] = i;
+    }
     *n_compute = n;
+    if (sidx) sidx[N] = ns;   // optional list of skipped candidates, its count after it
   }
 }
 
@@ -374,15 +379,15 @@ __global__ void score_finalize_kernel(const float* __restrict__ partials, int nc
 // Used by cs_search_step.  Two launches, no grid-wide barrier:
 //  drift_decide  every CTA takes a contiguous range of (candidate, chunk) items and
 //                writes their drift partials (x read with an L2 evict-last hint, so the
-//                skip update finds it in L2).  Per candidate, an arrival counter records
-//                how many of its chunks are done; the CTA that completes a candidate
-//                takes its decision (the same fixed-order sum of the same partials as
-//                the two-pass form, so the same bits), and the CTA that completes the
-//                last decision writes the compaction list.  Counters are left at zero.
+//                skip update finds it in L2), then counts itself in on one arrival
+//                counter.  The CTA that arrives last takes every decision (one warp per
+//                candidate, the same fixed-order sum of the same partials as the two-pass
+//                form, so the same bits), writes the lists of computing and skipped
+//                candidates and leaves the counter at zero.
 //  skip_update   launched with programmatic stream serialisation: its CTAs are
 //                scheduled while the first kernel drains and wait (griddepcontrol.wait)
-//                for its completion; each walks the same item range newest chunk first
-//                and applies Eq. skip + Eq. euler to skipped candidates.
+//                for its completion, then spread the skipped candidates' chunks over
+//                the grid and apply Eq. skip + Eq. euler.
 // No CTA ever waits for another CTA, so neither kernel needs co-resident CTAs.
 
 __device__ __forceinline__ void pdl_launch_dependents() {
@@ -390,8 +395,9 @@ __device__ __forceinline__ void pdl_launch_dependents() {
 }
 __device__ __forceinline__ void pdl_wait_primary() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
-// The decision of one candidate from its chunk partials (one warp; lane 0 writes).
-// Identical arithmetic to decide_finalize_kernel.  Returns 1 = compute (lane 0 only).
+// The decision of one candidate from its chunk partials (one warp; lane 0 writes the
+// state, the skip mask and dec[i] = 1 when it computes).  Identical arithmetic to
+// decide_finalize_kernel.
 __device__ __forceinline__ void decide_one(int i, const float* __restrict__ partials, int nch, bool free_step,
                                            float a_before, bool had, float tau, const uint8_t* __restrict__ force,
                                            float* __restrict__ accum, uint8_t* __restrict__ has_ref,
@@ -399,11 +405,26 @@ __device__ __forceinline__ void decide_one(int i, const float* __restrict__ part
                                            int lane) {
   float num = 0.f, den = 0.f;
   if (free_step) {
-    // partials written by other CTAs: read through L2 (never from this SM's L1)
+    // partials written by other CTAs: read through L2 (never from this SM's L1).  Lane l
+    // adds chunks l, l + 32, ... in order, as warp_sum_partials_f32 does (adding the 0 of
+    // a missing chunk changes nothing), but with every load issued before the first add.
+    const float2* pp = reinterpret_cast<const float2*>(partials) + (long long)i * nch;
     float s0 = 0.f, s1 = 0.f;
-    for (int c = lane; c < nch; c += 32) {
-      s0 += __ldcg(partials + ((long long)i * nch + c) * 2 + 0);
-      s1 += __ldcg(partials + ((long long)i * nch + c) * 2 + 1);
+    if (nch <= 32 * 16) {
+      float2 v[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) v[u] = lane + 32 * u < nch ? __ldcg(pp + lane + 32 * u) : make_float2(0.f, 0.f);
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        s0 += v[u].x;
+        s1 += v[u].y;
+      }
+    } else {
+      for (int c = lane; c < nch; c += 32) {
+        const float2 v = __ldcg(pp + c);
+        s0 += v.x;
+        s1 += v.y;
+      }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -443,101 +464,94 @@ __device__ __forceinline__ void decide_one(int i, const float* __restrict__ part
 __global__ void __launch_bounds__(kCacheThreads) drift_decide_kernel(
     const float* __restrict__ x, const float* __restrict__ xr, float* __restrict__ accum,
     uint8_t* __restrict__ has_ref, int N, long long D, int nch, float tau, const uint8_t* __restrict__ force,
-    uint8_t* __restrict__ skip_mask, uint8_t* __restrict__ dec, int32_t* __restrict__ idx,
-    int32_t* __restrict__ n_compute, float* __restrict__ partials, unsigned* __restrict__ counters, int* err) {
+    uint8_t* __restrict__ skip_mask, int32_t* __restrict__ idx, int32_t* __restrict__ n_compute,
+    int32_t* __restrict__ sidx, float* __restrict__ partials, unsigned* __restrict__ counter, int* err) {
   __shared__ float red[2][32];
-  __shared__ int s_flag, s_had;
-  __shared__ float s_a;
+  __shared__ int s_last;
+  extern __shared__ uint8_t flags[];            // [N] decisions (1 = compute), in the deciding CTA
   pdl_launch_dependents();   // the skip-update grid may be scheduled as soon as every CTA runs
   const int items = N * nch;
   const int per = (items + gridDim.x - 1) / gridDim.x;
+  const int active = (items + per - 1) / per;   // CTAs that own items (the others return)
   const int it0 = blockIdx.x * per, it1 = min(items, it0 + per);
   if (it0 >= it1) return;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int i_first = it0 / nch, i_last = (it1 - 1) / nch;
-  for (int i = i_first; i <= i_last; ++i) {
-    const int lo = max(it0, i * nch), hi = min(it1, (i + 1) * nch);
-    // the candidate's state before this step: read by one thread before this CTA's
-    // arrival (so before the deciding CTA can rewrite it) and shared with the others
-    if (threadIdx.x == 0) {
-      s_had = has_ref[i] != 0;
-      s_a = accum[i];
-    }
-    block_sync();
-    const bool had = s_had != 0;
-    const float a_before = s_a;
-    if (had) {
-      for (int item = lo; item < hi; ++item) {
-        const int c = item - i * nch;
-        const long long clo = (long long)c * kChunkElems, chi = min(D, clo + kChunkElems);
-        const float* xi = x + (long long)i * D + clo;
-        const float* ri = xr + (long long)i * D + clo;
-        const int n8 = (int)((chi - clo) >> 3);
-        float v[2] = {0.f, 0.f};
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = kCacheThreads / 32;
+  for (int item = it0; item < it1; ++item) {
+    const int i = item / nch, c = item % nch;
+    // has_ref is rewritten only by the deciding CTA, after every CTA has arrived
+    if (!has_ref[i]) continue;                  // uniform over the CTA
+    const long long clo = (long long)c * kChunkElems, chi = min(D, clo + kChunkElems);
+    const float* xi = x + (long long)i * D + clo;
+    const float* ri = xr + (long long)i * D + clo;
+    const int n8 = (int)((chi - clo) >> 3);
+    float v[2] = {0.f, 0.f};
 #pragma unroll 4
-        for (int e = threadIdx.x; e < n8; e += kCacheThreads) {
-          const F8 a = ld8_keep(xi + 8 * e), b = ld8_once(ri + 8 * e);
+    for (int e = threadIdx.x; e < n8; e += kCacheThreads) {
+      const F8 a = ld8_keep(xi + 8 * e), b = ld8_once(ri + 8 * e);
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const float dd = a.v[j] - b.v[j];
-            v[0] += dd * dd;
-            v[1] += b.v[j] * b.v[j];
-          }
-        }
-        block_sum<2>(v, red);
-        if (threadIdx.x == 0) {
-          partials[((long long)i * nch + c) * 2 + 0] = v[0];
-          partials[((long long)i * nch + c) * 2 + 1] = v[1];
-        }
-        block_sync();
+      for (int j = 0; j < 8; ++j) {
+        const float dd = a.v[j] - b.v[j];
+        v[0] += dd * dd;
+        v[1] += b.v[j] * b.v[j];
       }
     }
-    // arrival: this CTA's chunks of candidate i are done
+    block_sum<2>(v, red);
     if (threadIdx.x == 0) {
-      __threadfence();
-      const unsigned old = atomicAdd(&counters[i], (unsigned)(hi - lo));
-      s_flag = old + (unsigned)(hi - lo) == (unsigned)nch;
-    }
-    block_sync();
-    if (!s_flag) continue;
-    // this CTA completed candidate i: decide it
-    if (warp == 0) {
-      __threadfence();
-      decide_one(i, partials, nch, had, a_before, had, tau, force, accum, has_ref, skip_mask, dec, err, lane);
-      if (lane == 0) counters[i] = 0u;
-    }
-    block_sync();
-    if (threadIdx.x == 0) {
-      __threadfence();
-      s_flag = atomicAdd(&counters[N], 1u) == (unsigned)(N - 1);
-    }
-    block_sync();
-    if (s_flag && threadIdx.x == 0) {   // every candidate is decided: the compaction list
-      __threadfence();
-      const volatile uint8_t* dv = dec;
-      int n = 0;
-      for (int k = 0; k < N; ++k)
-        if (dv[k]) idx[n++] = k;
-      *n_compute = n;
-      counters[N] = 0u;
+      partials[((long long)i * nch + c) * 2 + 0] = v[0];
+      partials[((long long)i * nch + c) * 2 + 1] = v[1];
     }
     block_sync();
   }
+  // arrival: the CTA that arrives last takes every decision
+  if (threadIdx.x == 0) {
+    __threadfence();
+    s_last = atomicAdd(counter, 1u) == (unsigned)(active - 1);
+  }
+  block_sync();
+  if (!s_last) return;
+  __threadfence();
+  for (int i = warp; i < N; i += nw) {
+    const bool had = has_ref[i] != 0;
+    decide_one(i, partials, nch, had, accum[i], had, tau, force, accum, has_ref, skip_mask, flags, err, lane);
+  }
+  block_sync();
+  // compaction lists (computing candidates in idx, skipped ones in sidx, count after them)
+  if (warp == 0) {
+    int nc = 0, ns = 0;
+    for (int base = 0; base < N; base += 32) {
+      const int k = base + lane;
+      const bool valid = k < N;
+      const bool comp = valid && flags[k];
+      const unsigned bc = __ballot_sync(0xffffffffu, comp), bs = __ballot_sync(0xffffffffu, valid && !comp);
+      const unsigned below = (1u << lane) - 1u;
+      if (comp) idx[nc + __popc(bc & below)] = k;
+      if (valid && !comp) sidx[ns + __popc(bs & below)] = k;
+      nc += __popc(bc);
+      ns += __popc(bs);
+    }
+    if (lane == 0) {
+      *n_compute = nc;
+      sidx[N] = ns;
+      *counter = 0u;                            // ready for the next call
+    }
+  }
 }
 
-// Skipped candidates of the same item ranges: x += h (x + Delta), newest chunks first.
+// Skipped candidates: x += h (x + Delta).  The (skipped candidate, chunk) items, taken
+// from the list the deciding CTA wrote (sidx[0..n), n = sidx[N]), are spread evenly over
+// the grid, the last ones first (the latents the drift pass read last are the likeliest
+// to be still in L2).
 template <bool kScore>
 __global__ void __launch_bounds__(kCacheThreads) skip_update_kernel(
-    float* __restrict__ x, const float* __restrict__ delta, const uint8_t* __restrict__ skip_mask, int N, long long D,
+    float* __restrict__ x, const float* __restrict__ delta, const int32_t* __restrict__ sidx, int N, long long D,
     int nch, float h, float t_next, const float* __restrict__ target, float* __restrict__ spart) {
   __shared__ float red[1][32];
   pdl_wait_primary();        // the decisions (and every write of the first kernel) are visible
-  const int items = N * nch;
+  const int items = sidx[N] * nch;
   const int per = (items + gridDim.x - 1) / gridDim.x;
-  const int it0 = blockIdx.x * per, it1 = min(items, it0 + per);
+  const int it1 = items - blockIdx.x * per, it0 = max(0, it1 - per);
   for (int item = it1 - 1; item >= it0; --item) {
-    const int i = item / nch, c = item % nch;
-    if (!skip_mask[i]) continue;
+    const int i = sidx[item / nch], c = item % nch;
     const long long lo = (long long)c * kChunkElems, hi = min(D, lo + kChunkElems);
     float* xi = x + (long long)i * D + lo;
     const float* di = delta + (long long)i * D + lo;
@@ -757,14 +771,15 @@ __global__ void __launch_bounds__(kCacheThreads) beam_refill_kernel(
 using namespace cs;
 
 // Workspace layout: drift partials [N][nch][2], score partials [N][nch], then (at a
-// 256-byte boundary) the single-pass step's arrival counters [N + 1] and decisions [N].
+// 256-byte boundary) the single-pass step's arrival counter and the skipped candidates'
+// list with its count [N + 1].
 static size_t counters_offset(int N, long long D) {
   return ((size_t)N * cache_chunks(D) * 3 * sizeof(float) + 255) / 256 * 256;
 }
 
 extern "C" size_t cs_cache_workspace_bytes(int N, long long D) {
   if (N <= 0 || D <= 0) return 0;
-  return counters_offset(N, D) + (size_t)(N + 1) * sizeof(unsigned) + (size_t)N + 256;
+  return counters_offset(N, D) + sizeof(unsigned) + (size_t)(N + 1) * sizeof(int32_t) + 256;
 }
 
 extern "C" cs_status cs_cache_decide(const float* x, const float* x_ref, float* accum, uint8_t* has_ref, int N,
@@ -858,15 +873,14 @@ extern "C" cs_status cs_cache_apply_cfg(float* x, float* x_ref, float* delta, co
 
 namespace cs {
 
-// The single-pass decide + skip of cs_search_step.  counters: N + 1 arrival counters, zero
-// on entry (every completed call leaves them at zero; the model keeps its own set, zeroed
-// when allocated, at a place that does not depend on N), and dec: N decision bytes; both
-// nullptr: the set inside the workspace, whose counters are cleared first.
+// The single-pass decide + skip of cs_search_step.  sc.counter: the arrival counter, zero
+// on entry (every completed call leaves it at zero; the model keeps its own, zeroed when
+// allocated); sc.sidx: N + 1 ints (the skipped candidates and their count).
+// sc.counter == nullptr: the pair inside the workspace, whose counter is cleared first.
 cs_status decide_skip_run(float* x, const float* x_ref, const float* delta, float* accum, uint8_t* has_ref, int N,
                           long long D, int step_k, int T, float t_cur, float t_next, float tau, int K_w, int K_c,
                           const uint8_t* force, uint8_t* skip_mask, int32_t* idx, int32_t* n_compute,
-                          const float* target, void* workspace, unsigned* counters, uint8_t* dec, int* err,
-                          cudaStream_t stream) {
+                          const float* target, void* workspace, StepScratch sc, int* err, cudaStream_t stream) {
   const int nch = cache_chunks(D);
   const int wf = window_forced(step_k, T, K_w, K_c) ? 1 : 0;
   if (wf && !force) {
@@ -876,25 +890,29 @@ cs_status decide_skip_run(float* x, const float* x_ref, const float* delta, floa
   }
   float* partials = static_cast<float*>(workspace);
   float* spart = partials + (size_t)N * nch * 2;
-  const bool counters_zero = counters != nullptr;
-  if (!counters) {
-    counters = reinterpret_cast<unsigned*>(static_cast<char*>(workspace) + counters_offset(N, D));
-    dec = reinterpret_cast<uint8_t*>(counters + N + 1);
+  const bool counter_zero = sc.counter != nullptr;
+  if (!counter_zero) {
+    sc.counter = reinterpret_cast<unsigned*>(static_cast<char*>(workspace) + counters_offset(N, D));
+    sc.sidx = reinterpret_cast<int32_t*>(sc.counter + 1);
   }
   const int items = N * nch;
-  int grid = num_sms() * 4;   // 4 CTAs of 256 threads per SM keep enough 32-byte loads in flight
-  if (grid > items) grid = items;
+  // every chunk in flight at once: up to 8 CTAs of 256 threads per SM (no CTA waits for
+  // another, so the grid needs no co-residency)
+  int grid = num_sms() * 8;
   if (wf) {
     // forced mask inside the window: no drift is evaluated, one CTA decides
     decide_finalize_kernel<<<1, 1024, N, stream>>>(partials, nch, accum, has_ref, N, 1, tau, force, skip_mask, idx,
-                                                  n_compute, err);
+                                                  n_compute, err, sc.sidx);
     CS_LAUNCHED();
   } else {
-    if (!counters_zero) CS_CUDA(cudaMemsetAsync(counters, 0, (size_t)(N + 1) * sizeof(unsigned), stream));
-    drift_decide_kernel<<<grid, kCacheThreads, 0, stream>>>(x, x_ref, accum, has_ref, N, D, nch, tau, force,
-                                                           skip_mask, dec, idx, n_compute, partials, counters, err);
+    if (!counter_zero) CS_CUDA(cudaMemsetAsync(sc.counter, 0, sizeof(unsigned), stream));
+    const int g1 = grid < items ? grid : items;
+    drift_decide_kernel<<<g1, kCacheThreads, N, stream>>>(x, x_ref, accum, has_ref, N, D, nch, tau, force, skip_mask,
+                                                         idx, n_compute, sc.sidx, partials, sc.counter, err);
     CS_LAUNCHED();
   }
+  // the skip update's grid is sized before the decisions exist: CTAs without items return
+  if (grid > items) grid = items;
   const float h = t_next - t_cur;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
@@ -905,13 +923,34 @@ cs_status decide_skip_run(float* x, const float* x_ref, const float* delta, floa
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  const int32_t* sidx = sc.sidx;
   if (target)
-    CS_CUDA(cudaLaunchKernelEx(&cfg, skip_update_kernel<true>, x, delta, (const uint8_t*)skip_mask, N, D, nch, h,
-                               t_next, target, spart));
+    CS_CUDA(cudaLaunchKernelEx(&cfg, skip_update_kernel<true>, x, delta, sidx, N, D, nch, h, t_next, target, spart));
   else
-    CS_CUDA(cudaLaunchKernelEx(&cfg, skip_update_kernel<false>, x, delta, (const uint8_t*)skip_mask, N, D, nch, h,
-                               t_next, (const float*)nullptr, (float*)nullptr));
+    CS_CUDA(cudaLaunchKernelEx(&cfg, skip_update_kernel<false>, x, delta, sidx, N, D, nch, h, t_next,
+                               (const float*)nullptr, (float*)nullptr));
   CS_LAUNCHED();
+  return CS_OK;
+}
+
+// Load every cache kernel now (cudaFuncGetAttributes loads a kernel that lazy module
+// loading has not loaded yet), so that no search step pays for a first launch: the
+// decision pass and the skip update first run on the first free step, the scoring
+// variants on the last step of a search.
+cs_status load_cache_kernels() {
+  const void* fns[] = {
+      (const void*)drift_decide_kernel,          (const void*)skip_update_kernel<true>,
+      (const void*)skip_update_kernel<false>,    (const void*)velocity_update_kernel<true>,
+      (const void*)velocity_update_kernel<false>, (const void*)score_finalize_split_kernel,
+      (const void*)decide_finalize_kernel,       (const void*)decide_all_compute_kernel,
+      (const void*)drift_partials_kernel,        (const void*)apply_computed_kernel<true>,
+      (const void*)apply_computed_kernel<false>, (const void*)score_finalize_kernel,
+      (const void*)topk_kernel,                  (const void*)beam_refill_kernel,
+  };
+  for (const void* f : fns) {
+    cudaFuncAttributes a;
+    CS_CUDA(cudaFuncGetAttributes(&a, f));
+  }
   return CS_OK;
 }
 
@@ -966,7 +1005,7 @@ extern "C" cs_status cs_cache_decide_skip(float* x, const float* x_ref, const fl
                  (!target || (reinterpret_cast<uintptr_t>(target) & 31) == 0),
              "cs_cache_decide_skip: needs D %% 8 == 0 and 32-byte aligned tensors");
   return decide_skip_run(x, x_ref, delta, accum, has_ref, N, D, step_k, T, t_cur, t_next, tau, K_w, K_c, force,
-                         skip_mask, idx, n_compute, target, workspace, nullptr, nullptr, err, stream);
+                         skip_mask, idx, n_compute, target, workspace, StepScratch{}, err, stream);
 }
 
 extern "C" cs_status cs_cache_apply_tokens(float* x, float* x_ref, float* delta, float* accum, uint8_t* has_ref,

@@ -34,19 +34,24 @@ cs_status unpatchify(const float* hout, const int32_t* idx, int n_c, int C, int 
                      long long idx_limit, int* err, cudaStream_t s);
 cs_status to_bf16_pad(const float* src, long long rows, int cols, int ld, __nv_bfloat16* dst, cudaStream_t s);
 
-// cache.cu: the single-pass decide + skip (counters: N + 1 arrival counters, zero on entry
-// and left zero, and dec: N decision bytes; both nullptr for the workspace's own set,
-// cleared by the call), and the computed update from the head's token output (spart:
-// the skipped candidates' score partials; tpart [N][F*H/2]).
+// cache.cu: the single-pass decide + skip and its small scratch (counter: the arrival
+// counter, zero on entry and left zero; sidx: N + 1 ints, the skipped candidates and their
+// count; both nullptr for the pair inside the workspace, cleared by the call), and the
+// computed update from the head's token output (spart: the skipped candidates' score
+// partials; tpart [N][F*H/2]).
+struct StepScratch {
+  unsigned* counter = nullptr;
+  int32_t* sidx = nullptr;
+};
 cs_status decide_skip_run(float* x, const float* x_ref, const float* delta, float* accum, uint8_t* has_ref, int N,
                           long long D, int step_k, int T, float t_cur, float t_next, float tau, int K_w, int K_c,
                           const uint8_t* force, uint8_t* skip_mask, int32_t* idx, int32_t* n_compute,
-                          const float* target, void* workspace, unsigned* counters, uint8_t* dec, int* err,
-                          cudaStream_t stream);
+                          const float* target, void* workspace, StepScratch sc, int* err, cudaStream_t stream);
 cs_status apply_tokens_run(float* x, float* x_ref, float* delta, float* accum, uint8_t* has_ref, uint8_t* skip_mask,
                            const float* hout, const int32_t* idx, int n_c, int N, int C, int F, int H, int W,
                            float t_cur, float t_next, const float* target, float* scores, const float* spart,
                            float* tpart, long long idx_limit, int* err, cudaStream_t stream);
 bool apply_tokens_supported(int C, int F, int H, int W);
+cs_status load_cache_kernels();
 
 }  // namespace cs

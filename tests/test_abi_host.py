@@ -45,8 +45,8 @@ def test_workspace_and_version(b):
     assert b.lib.cs_version().startswith(b"cachedsearch")
     # the default library has no index checks (that is lib/libcachedsearch_debug.so)
     assert b.lib.cs_build_flags() == (1 if os.environ.get("CS_LIBRARY_VARIANT") == "debug" else 0)
-    # partials (drift, score), then the single-pass step's counters [N + 1] and decisions [N]
-    assert b.cache_workspace_bytes(4, 2096640) == 4 * 256 * 12 + 5 * 4 + 4 + 256
+    # partials (drift, score), then the single-pass step's arrival counter and skipped list [N + 1]
+    assert b.cache_workspace_bytes(4, 2096640) == 4 * 256 * 12 + 4 + 5 * 4 + 256
     assert b.cache_workspace_bytes(0, 10) == 0
 
 
