@@ -158,6 +158,42 @@ bool valid_cfg(const cs_model_config* c) {
 
 }  // namespace
 
+// One run of the search step's cache kernels (both decision-pass kernels, with and without
+// scores, and the computed update) on scratch inside the residual-stream buffer, so that
+// the first free step of a search does not pay their first launch (measured on GB300: the
+// first decision pass of a process took ~25 us longer than the next one even with the
+// kernels loaded).  Leaves the model's counter at zero and its error word clear.
+static cs_status warm_cache_kernels(cs_model* m) {
+  const cs_model_config& c = m->cfg;
+  if (!m->tokens_update) return CS_OK;
+  const long long D = m->D;
+  float* x = m->resid;                      // 3 latents + a target + small state, all scratch
+  float* xr = x + D;
+  float* dl = xr + D;
+  float* y = dl + D;
+  float* small = y + D;                     // accum, scores, tile partials
+  uint8_t* bytes = reinterpret_cast<uint8_t*>(small + 8 + c.F * (c.H / 2));
+  uint8_t* has_ref = bytes;
+  uint8_t* skip = bytes + 16;
+  if ((size_t)(4 * D + 64 + c.F * (c.H / 2)) > (size_t)c.max_batch * m->L * c.d) return CS_OK;   // too small to hold it
+  CS_CUDA(cudaMemset(x, 0, (4 * D + 8 + c.F * (c.H / 2)) * sizeof(float) + 64));
+  for (int score = 0; score < 2; ++score) {
+    // a cached candidate far from a non-zero reference under an infinite threshold: a
+    // finite drift, and the candidate skips (the skip update runs)
+    CS_CUDA(cudaMemset(has_ref, 1, 1));
+    CS_CUDA(cudaMemset(xr, 0x3f, D * sizeof(float)));
+    CS_TRY(cs::decide_skip_run(x, xr, dl, small, has_ref, 1, D, 2, 3, 1.f, 0.5f, 1e30f, 0, 0, nullptr, skip, m->idx,
+                               m->n_compute, score ? y : nullptr, m->cache_ws,
+                               cs::StepScratch{m->cache_counter, m->cache_sidx}, m->err, 0));
+    CS_TRY(cs::apply_tokens_run(x, xr, dl, small, has_ref, skip, m->hout, m->idx_all, 1, 1, c.C, c.F, c.H, c.W, 1.f,
+                                0.5f, score ? y : nullptr, small + 1, reinterpret_cast<float*>(m->cache_ws) + 2 * ((D + 8191) / 8192),
+                                small + 8, 1, m->err, 0));
+  }
+  CS_CUDA(cudaDeviceSynchronize());
+  CS_CUDA(cudaMemset(m->err, 0, sizeof(int)));
+  return CS_OK;
+}
+
 extern "C" size_t cs_param_count(const cs_model_config* c) {
   if (!valid_cfg(c)) return 0;
   const size_t d = c->d, P = 4 * (size_t)c->C, F = c->ffn;
@@ -289,7 +325,7 @@ extern "C" cs_status cs_init_model(const cs_model_config* cfg, cs_model** out) {
   for (int i = 0; i < cfg->max_batch; ++i) iota[i] = i;
   cudaMemcpy(m->idx_all, iota.data(), iota.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
   m->tokens_update = cs::apply_tokens_supported(cfg->C, cfg->F, cfg->H, cfg->W);
-  if (cs::load_cache_kernels() != CS_OK) {
+  if (cs::load_cache_kernels() != CS_OK || warm_cache_kernels(m) != CS_OK) {
     cudaFree(m->ws);
     cudaFree(m->wmem);
     delete m;

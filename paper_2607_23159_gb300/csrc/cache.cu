@@ -14,6 +14,7 @@
 #include <cmath>
 #include <cstdint>
 #include <mutex>
+#include <vector>
 
 #include "common.cuh"
 #include "elementwise.h"
@@ -485,14 +486,32 @@ __global__ void __launch_bounds__(kCacheThreads) drift_decide_kernel(
     const float* ri = xr + (long long)i * D + clo;
     const int n8 = (int)((chi - clo) >> 3);
     float v[2] = {0.f, 0.f};
-#pragma unroll 4
-    for (int e = threadIdx.x; e < n8; e += kCacheThreads) {
-      const F8 a = ld8_keep(xi + 8 * e), b = ld8_once(ri + 8 * e);
+    if (n8 == 4 * kCacheThreads) {
+      // a full chunk: all eight 32-byte loads of the thread issued before the first use
+      // (the compiler left only part of them in flight, which cost ~4 us at N = 4)
+      F8 a[4], b[4];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const float dd = a.v[j] - b.v[j];
-        v[0] += dd * dd;
-        v[1] += b.v[j] * b.v[j];
+      for (int u = 0; u < 4; ++u) {
+        a[u] = ld8_keep(xi + 8 * (threadIdx.x + u * kCacheThreads));
+        b[u] = ld8_once(ri + 8 * (threadIdx.x + u * kCacheThreads));
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float dd = a[u].v[j] - b[u].v[j];
+          v[0] += dd * dd;
+          v[1] += b[u].v[j] * b[u].v[j];
+        }
+    } else {
+      for (int e = threadIdx.x; e < n8; e += kCacheThreads) {
+        const F8 a = ld8_keep(xi + 8 * e), b = ld8_once(ri + 8 * e);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float dd = a.v[j] - b.v[j];
+          v[0] += dd * dd;
+          v[1] += b.v[j] * b.v[j];
+        }
       }
     }
     block_sum<2>(v, red);
@@ -542,7 +561,7 @@ __global__ void __launch_bounds__(kCacheThreads) drift_decide_kernel(
 // the grid, the last ones first (the latents the drift pass read last are the likeliest
 // to be still in L2).
 template <bool kScore>
-__global__ void __launch_bounds__(kCacheThreads) skip_update_kernel(
+__global__ void __launch_bounds__(kCacheThreads, 4) skip_update_kernel(
     float* __restrict__ x, const float* __restrict__ delta, const int32_t* __restrict__ sidx, int N, long long D,
     int nch, float h, float t_next, const float* __restrict__ target, float* __restrict__ spart) {
   __shared__ float red[1][32];
@@ -558,6 +577,24 @@ __global__ void __launch_bounds__(kCacheThreads) skip_update_kernel(
     const float* yi = kScore ? target + lo : nullptr;
     const int n8 = (int)((hi - lo) >> 3);
     float acc[1] = {0.f};
+    if (!kScore && n8 == 4 * kCacheThreads) {   // a full chunk: all eight 32-byte loads in flight
+      F8 xa[4], da[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        xa[u] = ld8_once(xi + 8 * (threadIdx.x + u * kCacheThreads));
+        da[u] = ld8_once(di + 8 * (threadIdx.x + u * kCacheThreads));
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        float xn[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) xn[j] = xa[u].v[j] + h * (xa[u].v[j] + da[u].v[j]);   // Eq. skip + Eq. euler
+        float4* o4 = reinterpret_cast<float4*>(xi + 8 * (threadIdx.x + u * kCacheThreads));
+        __stcs(o4, make_float4(xn[0], xn[1], xn[2], xn[3]));
+        __stcs(o4 + 1, make_float4(xn[4], xn[5], xn[6], xn[7]));
+      }
+      continue;
+    }
 #pragma unroll 4
     for (int e = threadIdx.x; e < n8; e += kCacheThreads) {   // a chunk's four rounds of loads all in flight
       const F8 xv = ld8_once(xi + 8 * e), dv = ld8_once(di + 8 * e);
@@ -873,6 +910,24 @@ extern "C" cs_status cs_cache_apply_cfg(float* x, float* x_ref, float* delta, co
 
 namespace cs {
 
+// CTAs of 256 threads that fit on all SMs at once for `kernel` (dynamic shared memory
+// `smem` bytes), looked up once per (kernel, smem).
+static int resident_grid(const void* kernel, int smem) {
+  static std::mutex mu;
+  static std::vector<std::pair<std::pair<const void*, int>, int>> known;
+  std::lock_guard<std::mutex> lock(mu);
+  for (auto& k : known)
+    if (k.first.first == kernel && k.first.second == smem) return k.second;
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kCacheThreads, smem) != cudaSuccess || per_sm < 1) {
+    (void)cudaGetLastError();
+    per_sm = 4;
+  }
+  const int g = per_sm * num_sms();
+  known.push_back({{kernel, smem}, g});
+  return g;
+}
+
 // The single-pass decide + skip of cs_search_step.  sc.counter: the arrival counter, zero
 // on entry (every completed call leaves it at zero; the model keeps its own, zeroed when
 // allocated); sc.sidx: N + 1 ints (the skipped candidates and their count).
@@ -896,9 +951,11 @@ cs_status decide_skip_run(float* x, const float* x_ref, const float* delta, floa
     sc.sidx = reinterpret_cast<int32_t*>(sc.counter + 1);
   }
   const int items = N * nch;
-  // every chunk in flight at once: up to 8 CTAs of 256 threads per SM (no CTA waits for
-  // another, so the grid needs no co-residency)
-  int grid = num_sms() * 8;
+  // one wave of CTAs, each taking a contiguous range of chunks: a grid larger than what
+  // fits on the SMs at once leaves a second, partial wave that ends late (measured on
+  // GB300: 1024 one-chunk CTAs at 5 per SM took 14.6 us for what 512 two-chunk CTAs move
+  // in about 10); no CTA waits for another, so residency is a speed matter only
+  int grid = resident_grid((const void*)drift_decide_kernel, N);
   if (wf) {
     // forced mask inside the window: no drift is evaluated, one CTA decides
     decide_finalize_kernel<<<1, 1024, N, stream>>>(partials, nch, accum, has_ref, N, 1, tau, force, skip_mask, idx,
@@ -906,12 +963,13 @@ cs_status decide_skip_run(float* x, const float* x_ref, const float* delta, floa
     CS_LAUNCHED();
   } else {
     if (!counter_zero) CS_CUDA(cudaMemsetAsync(sc.counter, 0, sizeof(unsigned), stream));
-    const int g1 = grid < items ? grid : items;
+    const int g1 = grid < items ? grid : items;   // contiguous ranges of items/g1 chunks
     drift_decide_kernel<<<g1, kCacheThreads, N, stream>>>(x, x_ref, accum, has_ref, N, D, nch, tau, force, skip_mask,
                                                          idx, n_compute, sc.sidx, partials, sc.counter, err);
     CS_LAUNCHED();
   }
   // the skip update's grid is sized before the decisions exist: CTAs without items return
+  grid = resident_grid(target ? (const void*)skip_update_kernel<true> : (const void*)skip_update_kernel<false>, 0);
   if (grid > items) grid = items;
   const float h = t_next - t_cur;
   cudaLaunchConfig_t cfg = {};
