@@ -28,6 +28,12 @@
 // TMEM (512 columns): S_A [0,128), S_B [128,256) (P_g, all 128 keys packed in pairs, aliases
 // columns [0, 64) of S_g: one 64-column store), O_A [256, 256+hd), O_B [256+hd, 256+2hd).  V is stored
 // transposed (V^T [hd][keys]) so that it is a K-major B operand in shared memory.
+//
+// Two launch forms of the same per-item arithmetic: one item (256 query rows of one
+// (batch item, head)) per CTA for long key loops (self-attention), and a persistent form
+// (attn_body_persist) for short ones (cross-attention over the 512 text tokens), where an
+// item's fixed costs -- its Q load, first scores and O epilogue -- are as long as its key
+// loop and overlap the neighbouring items' work instead.  Both give the same bits.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -67,11 +73,10 @@ struct AttnCfg {
   static constexpr uint32_t IDESC_O = idesc_bf16_f32(128, HD);
 };
 
-template <int HD, bool TMA_O>
+template <int HD>
 __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensorMap& tmK, const CUtensorMap& tmV,
-                                          const CUtensorMap& tmO, const AttnArgs& p) {
+                                          const AttnArgs& p) {
   using Cfg = AttnCfg<HD>;
-  static_assert(!TMA_O || HD % 64 == 0, "TMA output boxes are 64 columns wide");
   constexpr int NS = Cfg::NSTAGE;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -86,8 +91,7 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensor
   uint64_t* o_done = p_full + 2;           // [2]
   uint64_t* tok = o_done + 2;              // [2]: tok[g] = tile g may start its next MMA group
   uint64_t* teardown = tok + 2;            // [2]
-  uint64_t* o_staged = teardown + 2;       // [2] (TMA_O): tile g's normalised O is in shared memory
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_staged + (TMA_O ? 2 : 0));
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(teardown + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -113,7 +117,6 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensor
     for (int g = 0; g < 2; ++g) {
       mbar_init(&tok[g], 1);
       mbar_init(&teardown[g], 1);
-      if (TMA_O) mbar_init(&o_staged[g], 128);
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -324,42 +327,7 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensor
     }
     // final: O / l -> bf16
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait_suspend(&o_done[g], (nt - 1) & 1, abort_flag, p.err));
-    if constexpr (TMA_O) {
-      // Rows go through the tile's own Q buffer (every MMA that read it has completed: the
-      // last o_done commit covers them) in the 128-byte-swizzled layout of a TMA box of
-      // 64 columns x 128 rows; one thread of the tile then stores the boxes (rows past Lq
-      // are clipped by the tensor map).
-      uint8_t* stg = sQ + g * Cfg::Q_BYTES;
-      if (ok) {
-        tc_fence_after();
-        const float inv_l = 1.f / l_run;
-#pragma unroll 1
-        for (int c = 0; c < HD / 32; ++c) {
-          uint32_t u[32];
-          tmem_ld32(tO + c * 32, u);
-          uint8_t* rowp = stg + (c >> 1) * Cfg::CH_BYTES + r * 128;
-#pragma unroll
-          for (int w = 0; w < 4; ++w) {
-            uint4 o4;
-            o4.x = pack_bf16x2(__uint_as_float(u[8 * w + 0]) * inv_l, __uint_as_float(u[8 * w + 1]) * inv_l);
-            o4.y = pack_bf16x2(__uint_as_float(u[8 * w + 2]) * inv_l, __uint_as_float(u[8 * w + 3]) * inv_l);
-            o4.z = pack_bf16x2(__uint_as_float(u[8 * w + 4]) * inv_l, __uint_as_float(u[8 * w + 5]) * inv_l);
-            o4.w = pack_bf16x2(__uint_as_float(u[8 * w + 6]) * inv_l, __uint_as_float(u[8 * w + 7]) * inv_l);
-            const int unit = (c & 1) * 4 + w;
-            *reinterpret_cast<uint4*>(rowp + ((unit ^ (r & 7)) << 4)) = o4;
-          }
-        }
-        fence_proxy_async_smem();
-        mbar_arrive(&o_staged[g]);
-        if (qtr == 0 && lane == 0 && q0 + g * 128 < p.Lq && mbar_wait(&o_staged[g], 0, abort_flag, p.err)) {
-#pragma unroll
-          for (int c2 = 0; c2 < HD / 64; ++c2)
-            tma_store_3d(&tmO, stg + c2 * Cfg::CH_BYTES, head * HD + c2 * 64, q0 + g * 128, jb);
-          bulk_commit();
-          bulk_wait_all();   // the writes are done before the CTA's shared memory goes away
-        }
-      }
-    } else if (ok) {
+    if (ok) {
       tc_fence_after();
       const int q = q0 + g * 128 + r;
       const float inv_l = 1.f / l_run;
@@ -392,20 +360,328 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensor
   }
 }
 
-// Two entry points so that the kernel with per-thread O stores keeps its three tensor maps.
+// Persistent form: one CTA per SM walks the items (256 query rows of one (batch item,
+// head)) it, it + G, ... (G = grid size) and keeps every pipeline running across item
+// boundaries: the K/V ring, the MMA token between the two issuers, and the barrier phases
+// continue, the producer loads the next item's Q as soon as the last score MMAs of the
+// current item have read theirs, and each softmax warp's O epilogue of one item overlaps
+// the next item's Q load and first score MMAs.  Every item runs the same arithmetic in the
+// same order as in the one-item-per-CTA kernel.
+template <int HD>
+__device__ __forceinline__ void attn_body_persist(const CUtensorMap& tmQ, const CUtensorMap& tmK, const CUtensorMap& tmV,
+                                                  const AttnArgs& p) {
+  using Cfg = AttnCfg<HD>;
+  constexpr int NS = Cfg::NSTAGE;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = smem;
+  uint8_t* sKV = sQ + 2 * Cfg::Q_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + NS * 2 * Cfg::SLOT);
+  uint64_t* q_full = bars;
+  uint64_t* kv_full = bars + 1;            // [NS]
+  uint64_t* kv_empty = kv_full + NS;       // [NS]
+  uint64_t* s_full = kv_empty + NS;        // [2]
+  uint64_t* p_full = s_full + 2;           // [2]
+  uint64_t* o_done = p_full + 2;           // [2]
+  uint64_t* tok = o_done + 2;              // [2]
+  uint64_t* teardown = tok + 2;            // [2]
+  uint64_t* q_empty = teardown + 2;        // both issuers' last score MMAs of an item are done
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_empty + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nqp = (p.Lq + 255) / 256;
+  const int items = nqp * p.B * p.heads;
+  const int nt = (p.Lk + Cfg::BKV - 1) / Cfg::BKV;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    mbar_init(q_empty, 2);
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 2);
+    }
+    for (int g = 0; g < 2; ++g) {
+      mbar_init(&s_full[g], 1);
+      mbar_init(&p_full[g], 128);
+      mbar_init(&o_done[g], 1);
+      mbar_init(&tok[g], 1);
+      mbar_init(&teardown[g], 1);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  block_sync();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  auto item_bh = [&](int it) { return it / nqp; };
+  auto item_q0 = [&](int it) { return (it % nqp) * 256; };
+  auto item_bkv = [&](int it) {
+    const int bh = item_bh(it), head = bh % p.heads, jb = bh / p.heads;
+    int kv_set = p.kv_shared && p.item_idx ? p.item_idx[jb] / p.x_rows : 0;
+    if (!index_ok(kv_set, p.kv_sets, p.err)) kv_set = 0;
+    return !p.kv_shared ? bh : kv_set * p.heads + head;
+  };
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tmQ);
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      int gst = 0, issued = 0, n = 0, q_issued = 0;
+      bool ok = true;
+      for (int it = blockIdx.x; ok && it < items; it += gridDim.x, ++n) {
+        const int bh = item_bh(it), q0 = item_q0(it), bkv = item_bkv(it);
+        // the previous item's score MMAs have read its Q
+        if (n > 0 && !mbar_wait(q_empty, (n - 1) & 1, abort_flag, p.err)) break;
+        ++q_issued;
+        mbar_arrive_expect_tx(q_full, 2 * Cfg::Q_BYTES);
+        for (int g = 0; g < 2; ++g)
+          for (int c = 0; c < Cfg::QCH; ++c)
+            tma_load_3d(sQ + g * Cfg::Q_BYTES + c * Cfg::CH_BYTES, &tmQ, q_full, c * 64, q0 + g * 128, bh);
+        for (int st = 0; st <= nt; ++st, ++gst) {
+          const int b = gst % NS;
+          if (!mbar_wait(&kv_empty[b], ((gst / NS) & 1) ^ 1, abort_flag, p.err)) { ok = false; break; }
+          uint8_t* dv = sKV + b * 2 * Cfg::SLOT;
+          uint8_t* dk = dv + Cfg::SLOT;
+          mbar_arrive_expect_tx(&kv_full[b], (st >= 1 ? Cfg::V_BYTES : 0) + (st < nt ? Cfg::K_BYTES : 0));
+          if (st < nt)
+            for (int c = 0; c < Cfg::QCH; ++c)
+              tma_load_3d(dk + c * Cfg::CH_BYTES, &tmK, &kv_full[b], c * 64, st * Cfg::BKV, bkv);
+          if (st >= 1)
+            for (int c = 0; c < 2; ++c)
+              tma_load_3d(dv + c * Cfg::VCH_BYTES, &tmV, &kv_full[b], (st - 1) * Cfg::BKV + c * 64, 0, bkv);
+          issued = gst + 1;
+        }
+      }
+      if (*abort_flag) {
+        // the loads of the last ring's worth of stages and of the last Q (bounded waits)
+        if (q_issued > 0) mbar_wait_teardown(q_full, (q_issued - 1) & 1);
+        for (int st = issued - NS < 0 ? 0 : issued - NS; st < issued; ++st)
+          mbar_wait_teardown(&kv_full[st % NS], (st / NS) & 1);
+      }
+    }
+  } else if (warp == 1 || warp == Cfg::ISSUER_B) {
+    // ------------------------------------------------------------ MMA issuers
+    // The same groups as the one-item kernel, in one continuous stream:
+    //   S_A(0) S_B(0) | PV_A(0) S_A(1) | PV_B(0) S_B(1) | ... | PV_A(nt-1) | PV_B(nt-1) | next item S_A(0) ...
+    // with the token handed over inside every group except the CTA's very last one.
+    if (lane == 0) {
+      const int g = warp == 1 ? 0 : 1;
+      const uint32_t q_base = smem_u32(sQ);
+      const uint32_t sdst = tmem_base + g * 128, odst = tmem_base + 256 + g * HD;
+      const uint64_t ad = sdesc_sw128(q_base + g * Cfg::Q_BYTES);
+      static_assert(Cfg::NSTAGE == 2 && Cfg::HANDOVER == 4, "descriptor tables: two stages, hand-over at 4");
+      constexpr int NKS = Cfg::HDS / 16;
+      auto v_addr = [&](int st) { return smem_u32(sKV + (st % NS) * 2 * Cfg::SLOT); };
+      auto k_addr = [&](int st) { return v_addr(st) + Cfg::SLOT; };
+      uint64_t qa[8], kb0[8], kb1[8], vb0[8], vb1[8];
+      uint32_t pa[8];
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint64_t offk = (uint64_t)(((kk >> 2) * Cfg::CH_BYTES + (kk & 3) * 32) >> 4);
+        const uint64_t offv = (uint64_t)(((kk >> 2) * Cfg::VCH_BYTES + (kk & 3) * 32) >> 4);
+        qa[kk] = ad + offk;
+        kb0[kk] = sdesc_sw128(k_addr(0)) + offk;
+        kb1[kk] = sdesc_sw128(k_addr(1)) + offk;
+        vb0[kk] = sdesc_sw128(v_addr(0)) + offv;
+        vb1[kk] = sdesc_sw128(v_addr(1)) + offv;
+        pa[kk] = sdst + kk * 8;
+      }
+      auto issue_s = [&](const uint64_t* kb, uint64_t* pass) {
+        if (pass && NKS == Cfg::HANDOVER) mbar_arrive(pass);
+        umma4_ss(sdst, qa, kb, Cfg::IDESC_S, 0u);
+        if (NKS == 8) {
+          if (pass) mbar_arrive(pass);
+          umma4_ss(sdst, qa + 4, kb + 4, Cfg::IDESC_S, 1u);
+        }
+        umma_commit(&s_full[g]);
+      };
+      auto issue_pv = [&](const uint64_t* vb, int j, uint64_t* pass) {
+        umma4_ts(odst, pa, vb, Cfg::IDESC_O, j > 0 ? 1u : 0u);
+        if (pass) mbar_arrive(pass);
+        umma4_ts(odst, pa + 4, vb + 4, Cfg::IDESC_O, 1u);
+        umma_commit(&o_done[g]);
+      };
+      uint64_t* other = &tok[1 - g];
+      int gst = 0, n = 0, tw = 0, pw = 0;   // stage counter, items, token waits, P waits
+      bool ok = true;
+      for (int it = blockIdx.x; ok && it < items; it += gridDim.x, ++n) {
+        const bool last_item = it + (int)gridDim.x >= items;
+        const int base = gst;
+        if (!mbar_wait(q_full, n & 1, abort_flag, p.err)) { ok = false; break; }
+        // S(0): tile A of the CTA's first item starts the stream, every other group waits its turn
+        if (!(g == 0 && n == 0)) {
+          if (!mbar_wait(&tok[g], tw & 1, abort_flag, p.err)) { ok = false; break; }
+          ++tw;
+        }
+        if (!mbar_wait(&kv_full[base % NS], (base / NS) & 1, abort_flag, p.err)) { ok = false; break; }
+        tc_fence_after();
+        issue_s((base % NS) == 0 ? kb0 : kb1, other);
+        if (nt == 1) umma_commit(q_empty);
+        umma_commit(&kv_empty[base % NS]);
+        for (int j = 0; j < nt; ++j) {
+          const int st = base + j + 1;
+          const bool more = j + 1 < nt;
+          if (!mbar_wait(&tok[g], tw & 1, abort_flag, p.err)) { ok = false; break; }
+          ++tw;
+          if (!mbar_wait(&kv_full[st % NS], (st / NS) & 1, abort_flag, p.err)) { ok = false; break; }
+          if (!mbar_wait(&p_full[g], pw & 1, abort_flag, p.err)) { ok = false; break; }
+          ++pw;
+          tc_fence_after();
+          // every group hands the token over, except tile B's last group of the CTA's last item
+          uint64_t* pass = (g == 1 && !more && last_item) ? nullptr : other;
+          if ((st % NS) == 0) {
+            issue_pv(vb0, j, more ? nullptr : pass);
+            if (more) issue_s(kb0, pass);
+          } else {
+            issue_pv(vb1, j, more ? nullptr : pass);
+            if (more) issue_s(kb1, pass);
+          }
+          if (more && j + 2 == nt) umma_commit(q_empty);   // this item's last score MMAs
+          umma_commit(&kv_empty[st % NS]);
+        }
+        gst = base + nt + 1;
+      }
+      if (*abort_flag) {
+        umma_commit(&teardown[g]);
+        mbar_wait_teardown(&teardown[g], 0);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ softmax + epilogue
+    const int g = (warp - 2) >> 2;
+    const int qtr = warp & 3;
+    const int r = qtr * 32 + lane;
+    const uint32_t lane_off = (uint32_t)(qtr * 32) << 16;
+    const uint32_t tS = tmem_base + lane_off + g * 128;
+    const uint32_t tO = tmem_base + lane_off + 256 + g * HD;
+    const float sl2 = p.scale_log2;
+    const uint64_t sc2 = f2_pack(sl2, sl2);
+    const int d = p.heads * HD;
+    int sc = 0;   // S tiles of this query tile consumed so far (all items)
+    bool ok = true;
+    for (int it = blockIdx.x; ok && it < items; it += gridDim.x) {
+      const int bh = item_bh(it), q0 = item_q0(it);
+      const int head = bh % p.heads, jb = bh / p.heads;
+      float m_run = -INFINITY, l_run = 0.f;
+      for (int j = 0; j < nt; ++j, ++sc) {
+        if (!__all_sync(0xffffffffu, mbar_wait_suspend(&s_full[g], sc & 1, abort_flag, p.err))) { ok = false; break; }
+        tc_fence_after();
+        uint32_t u[128];
+        float rmax;
+        const int valid = p.Lk - j * Cfg::BKV;
+        if (valid >= Cfg::BKV) {
+          tmem_ld128_max(tS, u, rmax);
+        } else {
+          tmem_ld128(tS, u);
+#pragma unroll
+          for (int e = 0; e < Cfg::BKV; ++e)
+            if (e >= valid) u[e] = __float_as_uint(-INFINITY);
+          float mx[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) mx[q] = __uint_as_float(u[q]);
+#pragma unroll
+          for (int e = 4; e < Cfg::BKV - 4; e += 8) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) mx[q] = fmax3(mx[q], __uint_as_float(u[e + 2 * q]), __uint_as_float(u[e + 2 * q + 1]));
+          }
+#pragma unroll
+          for (int q = 0; q < 4; ++q) mx[q] = fmaxf(mx[q], __uint_as_float(u[Cfg::BKV - 4 + q]));
+          rmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+        }
+        const float m_new = fmaxf(m_run, rmax * sl2);
+        const bool need = (j == 0) || (m_new > m_run + 8.f);
+        const bool warp_need = __any_sync(0xffffffffu, need);
+        const float m_use = need ? m_new : m_run;
+        const float factor = need ? ex2_approx(m_run - m_use) : 1.f;
+        const uint64_t nm2 = f2_pack(-m_use, -m_use);
+        uint64_t acc[2] = {0ull, 0ull};
+#pragma unroll
+        for (int i = 0; i < Cfg::BKV / 2; ++i) {
+          float a, b;
+          f2_unpack(f2_fma(f2_pack(__uint_as_float(u[2 * i]), __uint_as_float(u[2 * i + 1])), sc2, nm2), a, b);
+          a = ex2_approx(a);
+          b = ex2_approx(b);
+          acc[i & 1] = f2_add(acc[i & 1], f2_pack(a, b));
+          u[i] = pack_bf16x2(a, b);
+        }
+        float s0, s1, s2, s3;
+        f2_unpack(acc[0], s0, s1);
+        f2_unpack(acc[1], s2, s3);
+        l_run = l_run * factor + ((s0 + s1) + (s2 + s3));
+        m_run = m_use;
+        if (j > 0 && warp_need) {
+#pragma unroll 1
+          for (int c = 0; c < HD / 32; ++c) {
+            uint32_t o[32];
+            tmem_ld32(tO + c * 32, o);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * factor);
+            tmem_st32(tO + c * 32, o);
+          }
+        }
+        tmem_st64(tS, u);
+        tc_fence_before();
+        mbar_arrive(&p_full[g]);
+      }
+      if (!ok) break;
+      // epilogue: the item's last PV group (o_done phase sc - 1) has completed
+      if (!__all_sync(0xffffffffu, mbar_wait_suspend(&o_done[g], (sc - 1) & 1, abort_flag, p.err))) { ok = false; break; }
+      tc_fence_after();
+      const int q = q0 + g * 128 + r;
+      const float inv_l = 1.f / l_run;
+      __nv_bfloat16* orow = p.o + ((long long)jb * p.Lq + q) * d + head * HD;
+#pragma unroll 1
+      for (int c = 0; c < HD / 32; ++c) {
+        uint32_t u[32];
+        tmem_ld32(tO + c * 32, u);
+        if (q < p.Lq) {
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+            uint4 o4;
+            o4.x = pack_bf16x2(__uint_as_float(u[8 * w + 0]) * inv_l, __uint_as_float(u[8 * w + 1]) * inv_l);
+            o4.y = pack_bf16x2(__uint_as_float(u[8 * w + 2]) * inv_l, __uint_as_float(u[8 * w + 3]) * inv_l);
+            o4.z = pack_bf16x2(__uint_as_float(u[8 * w + 4]) * inv_l, __uint_as_float(u[8 * w + 5]) * inv_l);
+            o4.w = pack_bf16x2(__uint_as_float(u[8 * w + 6]) * inv_l, __uint_as_float(u[8 * w + 7]) * inv_l);
+            reinterpret_cast<uint4*>(orow + c * 32)[w] = o4;
+          }
+        }
+      }
+      // O is read before this warp's next arrival on p_full, which the next PV (that
+      // overwrites O) waits for: tmem_ld32 waits for its loads to complete
+    }
+  }
+
+  tc_fence_before();
+  block_sync();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, 512);
+  }
+}
+
+template <int HD>
+__global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
+    attn_tcgen05_persist_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                                const __grid_constant__ CUtensorMap tmV, const AttnArgs p) {
+  attn_body_persist<HD>(tmQ, tmK, tmV, p);
+}
+
 template <int HD>
 __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
     attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                         const __grid_constant__ CUtensorMap tmV, const AttnArgs p) {
-  attn_body<HD, false>(tmQ, tmK, tmV, tmQ, p);
+  attn_body<HD>(tmQ, tmK, tmV, p);
 }
-template <int HD>
-__global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
-    attn_tcgen05_tma_o_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                              const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
-                              const AttnArgs p) {
-  attn_body<HD, true>(tmQ, tmK, tmV, tmO, p);
-}
+
+constexpr int kPersistMaxKeys = 2048;
 
 template <int HD>
 static cs_status launch_attn(const void* q, const void* k, const void* vt, void* o, int B, int heads, int Lq, int Lk,
@@ -413,7 +689,7 @@ static cs_status launch_attn(const void* q, const void* k, const void* vt, void*
                              int* err, cudaStream_t stream) {
   using Cfg = AttnCfg<HD>;
   const int BH = B * heads, Bkv = kv_shared ? heads * kv_sets : BH;
-  CUtensorMap tq, tk, tv, to;
+  CUtensorMap tq, tk, tv;
   {
     const uint64_t dims[3] = {(uint64_t)Cfg::HDS, (uint64_t)Lq, (uint64_t)BH};
     const uint64_t str[2] = {(uint64_t)Cfg::HDS * 2, (uint64_t)Lq * Cfg::HDS * 2};
@@ -432,18 +708,6 @@ static cs_status launch_attn(const void* q, const void* k, const void* vt, void*
     const uint32_t box[3] = {64, (uint32_t)HD, 1};
     CS_TRY(make_tmap_bf16(&tv, vt, 3, dims, str, box));
   }
-  // O through TMA stores pays off when the key loop is short (cross-attention: the epilogue
-  // is a third of a CTA); with long key loops it measured slower (the kernel's registers
-  // are tight), so there each thread stores its own rows.
-  const bool tma_o = HD % 64 == 0 && Lk <= 2048;
-  to = tq;   // unused unless tma_o
-  if (tma_o) {
-    // O [B][Lq][heads*hd]: 64-column x 128-row boxes, clipped at Lq within each batch item
-    const uint64_t dims[3] = {(uint64_t)heads * HD, (uint64_t)Lq, (uint64_t)B};
-    const uint64_t str[2] = {(uint64_t)heads * HD * 2, (uint64_t)Lq * heads * HD * 2};
-    const uint32_t box[3] = {64, 128, 1};
-    CS_TRY(make_tmap_bf16(&to, o, 3, dims, str, box));
-  }
   AttnArgs a{};
   a.B = B; a.heads = heads; a.Lq = Lq; a.Lk = Lk; a.kv_shared = kv_shared;
   a.item_idx = item_idx; a.x_rows = x_rows > 0 ? x_rows : 1; a.kv_sets = kv_sets;
@@ -451,14 +715,17 @@ static cs_status launch_attn(const void* q, const void* k, const void* vt, void*
   a.o = static_cast<__nv_bfloat16*>(o);
   a.err = err;
   dim3 grid((Lq + 255) / 256, BH);
-  if constexpr (HD % 64 == 0) {
-    if (tma_o) {
-      auto kern = attn_tcgen05_tma_o_kernel<HD>;
-      CS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
-      kern<<<grid, Cfg::THREADS, Cfg::SMEM, stream>>>(tq, tk, tv, to, a);
-      CS_LAUNCHED();
-      return CS_OK;
-    }
+  if (Lk <= kPersistMaxKeys) {
+    // short key loops (cross-attention over the text): one CTA per SM walks the items, so
+    // that an item's Q load, first scores and O epilogue overlap its neighbours' work
+    // (measured at 4 x 12 x 32760 x 512: 973 -> 1026 TFLOP/s; at 32760 keys the same
+    // form measured 1-3 % slower than one item per CTA, so long key loops keep that)
+    auto kern = attn_tcgen05_persist_kernel<HD>;
+    CS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
+    const int items = grid.x * grid.y;
+    kern<<<items < num_sms() ? items : num_sms(), Cfg::THREADS, Cfg::SMEM, stream>>>(tq, tk, tv, a);
+    CS_LAUNCHED();
+    return CS_OK;
   }
   auto kern = attn_tcgen05_kernel<HD>;
   CS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));

@@ -167,11 +167,6 @@ __device__ __forceinline__ void tma_store_2d(const void* map, const void* src, i
                "r"(y), "r"(smem_u32(src))
                : "memory");
 }
-__device__ __forceinline__ void tma_store_3d(const void* map, const void* src, int x, int y, int z) {
-  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.tile.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(map),
-               "r"(x), "r"(y), "r"(z), "r"(smem_u32(src))
-               : "memory");
-}
 __device__ __forceinline__ void tma_reduce_add_2d(const void* map, const void* src, int x, int y) {
   asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.tile.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
                    map),
