@@ -34,7 +34,7 @@ for k in range(1, cfg.T + 1):
 torch.cuda.synchronize()
 out = {"checks": B.index_checks(), "x": hashlib.sha1(st["x"].cpu().numpy().tobytes()).hexdigest(),
        "masks": masks, "err": model.device_error()}
-if B.index_checks():     # only this build is given a bad index: it skips the access
+if B.index_checks():     # only the index-checking library is given a bad index: it skips the access
     v = torch.zeros(cfg.N, m.D, device="cuda")
     idx = torch.tensor([1, -1], dtype=torch.int32, device="cuda")
     model.dit_forward(st["x"], idx, 2, 0.5, v)
