@@ -73,6 +73,95 @@ struct AttnCfg {
   static constexpr uint32_t IDESC_O = idesc_bf16_f32(128, HD);
 };
 
+// One key tile of the online softmax of one query row (one thread per row, after S(j) of
+// its tile is complete): the scores of the tile from TMEM (keys past `valid` masked), the
+// running maximum and sum in log2 units, P = 2^(s * scale - m) written back as bf16 pairs over
+// the first 64 S columns, and O rescaled when the maximum grew by more than 8 (lazy rescale;
+// the PV of the previous tile has finished, since the commit that signalled S(j) covers it).
+template <int HD>
+__device__ __forceinline__ void softmax_tile(uint32_t tS, uint32_t tO, int j, int valid, float sl2, uint64_t sc2,
+                                             float& m_run, float& l_run) {
+  using Cfg = AttnCfg<HD>;
+  uint32_t u[128];
+  float rmax;
+  if (valid >= Cfg::BKV) {
+    tmem_ld128_max(tS, u, rmax);            // the row maximum comes with the load
+  } else {                                  // last, partial key tile: mask, then reduce
+    tmem_ld128(tS, u);
+#pragma unroll
+    for (int e = 0; e < Cfg::BKV; ++e)
+      if (e >= valid) u[e] = __float_as_uint(-INFINITY);
+    float mx[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) mx[q] = __uint_as_float(u[q]);
+#pragma unroll
+    for (int e = 4; e < Cfg::BKV - 4; e += 8) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) mx[q] = fmax3(mx[q], __uint_as_float(u[e + 2 * q]), __uint_as_float(u[e + 2 * q + 1]));
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) mx[q] = fmaxf(mx[q], __uint_as_float(u[Cfg::BKV - 4 + q]));
+    rmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+  }
+  const float m_new = fmaxf(m_run, rmax * sl2);
+  const bool need = (j == 0) || (m_new > m_run + 8.f);
+  const bool warp_need = __any_sync(0xffffffffu, need);
+  const float m_use = need ? m_new : m_run;
+  const float factor = need ? ex2_approx(m_run - m_use) : 1.f;
+  const uint64_t nm2 = f2_pack(-m_use, -m_use);
+  // p = 2^(s * scale * log2(e) - m) on pairs; P packed as bf16 pairs in place (u[0..63])
+  uint64_t acc[2] = {0ull, 0ull};
+#pragma unroll
+  for (int i = 0; i < Cfg::BKV / 2; ++i) {
+    float a, b;
+    f2_unpack(f2_fma(f2_pack(__uint_as_float(u[2 * i]), __uint_as_float(u[2 * i + 1])), sc2, nm2), a, b);
+    a = ex2_approx(a);
+    b = ex2_approx(b);
+    acc[i & 1] = f2_add(acc[i & 1], f2_pack(a, b));
+    u[i] = pack_bf16x2(a, b);
+  }
+  float s0, s1, s2, s3;
+  f2_unpack(acc[0], s0, s1);
+  f2_unpack(acc[1], s2, s3);
+  l_run = l_run * factor + ((s0 + s1) + (s2 + s3));
+  m_run = m_use;
+  // PV of the previous tile has finished: the commit that signalled S(j) also covers
+  // every MMA issued before it, so O may be rescaled and P overwritten now
+  if (j > 0 && warp_need) {
+#pragma unroll 1
+    for (int c = 0; c < HD / 32; ++c) {
+      uint32_t o[32];
+      tmem_ld32(tO + c * 32, o);
+#pragma unroll
+      for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * factor);
+      tmem_st32(tO + c * 32, o);
+    }
+  }
+  tmem_st64(tS, u);                         // P: keys 2c, 2c+1 packed in column c
+}
+
+// The normalised O row (O / l, bf16) of one query row from TMEM to memory.
+template <int HD>
+__device__ __forceinline__ void store_o_row(uint32_t tO, float l_run, __nv_bfloat16* orow, bool in_range) {
+  const float inv_l = 1.f / l_run;
+#pragma unroll 1
+  for (int c = 0; c < HD / 32; ++c) {
+    uint32_t u[32];
+    tmem_ld32(tO + c * 32, u);
+    if (in_range) {
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        uint4 o4;
+        o4.x = pack_bf16x2(__uint_as_float(u[8 * w + 0]) * inv_l, __uint_as_float(u[8 * w + 1]) * inv_l);
+        o4.y = pack_bf16x2(__uint_as_float(u[8 * w + 2]) * inv_l, __uint_as_float(u[8 * w + 3]) * inv_l);
+        o4.z = pack_bf16x2(__uint_as_float(u[8 * w + 4]) * inv_l, __uint_as_float(u[8 * w + 5]) * inv_l);
+        o4.w = pack_bf16x2(__uint_as_float(u[8 * w + 6]) * inv_l, __uint_as_float(u[8 * w + 7]) * inv_l);
+        reinterpret_cast<uint4*>(orow + c * 32)[w] = o4;
+      }
+    }
+  }
+}
+
 template <int HD>
 __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensorMap& tmK, const CUtensorMap& tmV,
                                           const AttnArgs& p) {
@@ -265,63 +354,7 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensor
     for (int j = 0; j < nt; ++j) {
       if (!__all_sync(0xffffffffu, mbar_wait_suspend(&s_full[g], j & 1, abort_flag, p.err))) { ok = false; break; }
       tc_fence_after();
-      uint32_t u[128];
-      float rmax;
-      const int valid = p.Lk - j * Cfg::BKV;
-      if (valid >= Cfg::BKV) {
-        tmem_ld128_max(tS, u, rmax);            // the row maximum comes with the load
-      } else {                                  // last, partial key tile: mask, then reduce
-        tmem_ld128(tS, u);
-#pragma unroll
-        for (int e = 0; e < Cfg::BKV; ++e)
-          if (e >= valid) u[e] = __float_as_uint(-INFINITY);
-        float mx[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) mx[q] = __uint_as_float(u[q]);
-#pragma unroll
-        for (int e = 4; e < Cfg::BKV - 4; e += 8) {
-#pragma unroll
-          for (int q = 0; q < 4; ++q) mx[q] = fmax3(mx[q], __uint_as_float(u[e + 2 * q]), __uint_as_float(u[e + 2 * q + 1]));
-        }
-#pragma unroll
-        for (int q = 0; q < 4; ++q) mx[q] = fmaxf(mx[q], __uint_as_float(u[Cfg::BKV - 4 + q]));
-        rmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
-      }
-      const float m_new = fmaxf(m_run, rmax * sl2);
-      const bool need = (j == 0) || (m_new > m_run + 8.f);
-      const bool warp_need = __any_sync(0xffffffffu, need);
-      const float m_use = need ? m_new : m_run;
-      const float factor = need ? ex2_approx(m_run - m_use) : 1.f;
-      const uint64_t nm2 = f2_pack(-m_use, -m_use);
-      // p = 2^(s * scale * log2(e) - m) on pairs; P packed as bf16 pairs in place (u[0..63])
-      uint64_t acc[2] = {0ull, 0ull};
-#pragma unroll
-      for (int i = 0; i < Cfg::BKV / 2; ++i) {
-        float a, b;
-        f2_unpack(f2_fma(f2_pack(__uint_as_float(u[2 * i]), __uint_as_float(u[2 * i + 1])), sc2, nm2), a, b);
-        a = ex2_approx(a);
-        b = ex2_approx(b);
-        acc[i & 1] = f2_add(acc[i & 1], f2_pack(a, b));
-        u[i] = pack_bf16x2(a, b);
-      }
-      float s0, s1, s2, s3;
-      f2_unpack(acc[0], s0, s1);
-      f2_unpack(acc[1], s2, s3);
-      l_run = l_run * factor + ((s0 + s1) + (s2 + s3));
-      m_run = m_use;
-      // PV of the previous tile has finished: the commit that signalled S(j) also covers
-      // every MMA issued before it, so O may be rescaled and P overwritten now
-      if (j > 0 && warp_need) {
-#pragma unroll 1
-        for (int c = 0; c < HD / 32; ++c) {
-          uint32_t o[32];
-          tmem_ld32(tO + c * 32, o);
-#pragma unroll
-          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * factor);
-          tmem_st32(tO + c * 32, o);
-        }
-      }
-      tmem_st64(tS, u);                         // P: keys 2c, 2c+1 packed in column c
+      softmax_tile<HD>(tS, tO, j, p.Lk - j * Cfg::BKV, sl2, sc2, m_run, l_run);
       tc_fence_before();
       mbar_arrive(&p_full[g]);
     }
@@ -330,25 +363,7 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tmQ, const CUtensor
     if (ok) {
       tc_fence_after();
       const int q = q0 + g * 128 + r;
-      const float inv_l = 1.f / l_run;
-      const int d = p.heads * HD;
-      __nv_bfloat16* orow = p.o + ((long long)jb * p.Lq + q) * d + head * HD;
-#pragma unroll 1
-      for (int c = 0; c < HD / 32; ++c) {
-        uint32_t u[32];
-        tmem_ld32(tO + c * 32, u);
-        if (q < p.Lq) {
-#pragma unroll
-          for (int w = 0; w < 4; ++w) {
-            uint4 o4;
-            o4.x = pack_bf16x2(__uint_as_float(u[8 * w + 0]) * inv_l, __uint_as_float(u[8 * w + 1]) * inv_l);
-            o4.y = pack_bf16x2(__uint_as_float(u[8 * w + 2]) * inv_l, __uint_as_float(u[8 * w + 3]) * inv_l);
-            o4.z = pack_bf16x2(__uint_as_float(u[8 * w + 4]) * inv_l, __uint_as_float(u[8 * w + 5]) * inv_l);
-            o4.w = pack_bf16x2(__uint_as_float(u[8 * w + 6]) * inv_l, __uint_as_float(u[8 * w + 7]) * inv_l);
-            reinterpret_cast<uint4*>(orow + c * 32)[w] = o4;
-          }
-        }
-      }
+      store_o_row<HD>(tO, l_run, p.o + ((long long)jb * p.Lq + q) * (p.heads * HD) + head * HD, q < p.Lq);
     }
   }
 
@@ -574,60 +589,7 @@ __device__ __forceinline__ void attn_body_persist(const CUtensorMap& tmQ, const 
       for (int j = 0; j < nt; ++j, ++sc) {
         if (!__all_sync(0xffffffffu, mbar_wait_suspend(&s_full[g], sc & 1, abort_flag, p.err))) { ok = false; break; }
         tc_fence_after();
-        uint32_t u[128];
-        float rmax;
-        const int valid = p.Lk - j * Cfg::BKV;
-        if (valid >= Cfg::BKV) {
-          tmem_ld128_max(tS, u, rmax);
-        } else {
-          tmem_ld128(tS, u);
-#pragma unroll
-          for (int e = 0; e < Cfg::BKV; ++e)
-            if (e >= valid) u[e] = __float_as_uint(-INFINITY);
-          float mx[4];
-#pragma unroll
-          for (int q = 0; q < 4; ++q) mx[q] = __uint_as_float(u[q]);
-#pragma unroll
-          for (int e = 4; e < Cfg::BKV - 4; e += 8) {
-#pragma unroll
-            for (int q = 0; q < 4; ++q) mx[q] = fmax3(mx[q], __uint_as_float(u[e + 2 * q]), __uint_as_float(u[e + 2 * q + 1]));
-          }
-#pragma unroll
-          for (int q = 0; q < 4; ++q) mx[q] = fmaxf(mx[q], __uint_as_float(u[Cfg::BKV - 4 + q]));
-          rmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
-        }
-        const float m_new = fmaxf(m_run, rmax * sl2);
-        const bool need = (j == 0) || (m_new > m_run + 8.f);
-        const bool warp_need = __any_sync(0xffffffffu, need);
-        const float m_use = need ? m_new : m_run;
-        const float factor = need ? ex2_approx(m_run - m_use) : 1.f;
-        const uint64_t nm2 = f2_pack(-m_use, -m_use);
-        uint64_t acc[2] = {0ull, 0ull};
-#pragma unroll
-        for (int i = 0; i < Cfg::BKV / 2; ++i) {
-          float a, b;
-          f2_unpack(f2_fma(f2_pack(__uint_as_float(u[2 * i]), __uint_as_float(u[2 * i + 1])), sc2, nm2), a, b);
-          a = ex2_approx(a);
-          b = ex2_approx(b);
-          acc[i & 1] = f2_add(acc[i & 1], f2_pack(a, b));
-          u[i] = pack_bf16x2(a, b);
-        }
-        float s0, s1, s2, s3;
-        f2_unpack(acc[0], s0, s1);
-        f2_unpack(acc[1], s2, s3);
-        l_run = l_run * factor + ((s0 + s1) + (s2 + s3));
-        m_run = m_use;
-        if (j > 0 && warp_need) {
-#pragma unroll 1
-          for (int c = 0; c < HD / 32; ++c) {
-            uint32_t o[32];
-            tmem_ld32(tO + c * 32, o);
-#pragma unroll
-            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * factor);
-            tmem_st32(tO + c * 32, o);
-          }
-        }
-        tmem_st64(tS, u);
+        softmax_tile<HD>(tS, tO, j, p.Lk - j * Cfg::BKV, sl2, sc2, m_run, l_run);
         tc_fence_before();
         mbar_arrive(&p_full[g]);
       }
@@ -636,24 +598,7 @@ __device__ __forceinline__ void attn_body_persist(const CUtensorMap& tmQ, const 
       if (!__all_sync(0xffffffffu, mbar_wait_suspend(&o_done[g], (sc - 1) & 1, abort_flag, p.err))) { ok = false; break; }
       tc_fence_after();
       const int q = q0 + g * 128 + r;
-      const float inv_l = 1.f / l_run;
-      __nv_bfloat16* orow = p.o + ((long long)jb * p.Lq + q) * d + head * HD;
-#pragma unroll 1
-      for (int c = 0; c < HD / 32; ++c) {
-        uint32_t u[32];
-        tmem_ld32(tO + c * 32, u);
-        if (q < p.Lq) {
-#pragma unroll
-          for (int w = 0; w < 4; ++w) {
-            uint4 o4;
-            o4.x = pack_bf16x2(__uint_as_float(u[8 * w + 0]) * inv_l, __uint_as_float(u[8 * w + 1]) * inv_l);
-            o4.y = pack_bf16x2(__uint_as_float(u[8 * w + 2]) * inv_l, __uint_as_float(u[8 * w + 3]) * inv_l);
-            o4.z = pack_bf16x2(__uint_as_float(u[8 * w + 4]) * inv_l, __uint_as_float(u[8 * w + 5]) * inv_l);
-            o4.w = pack_bf16x2(__uint_as_float(u[8 * w + 6]) * inv_l, __uint_as_float(u[8 * w + 7]) * inv_l);
-            reinterpret_cast<uint4*>(orow + c * 32)[w] = o4;
-          }
-        }
-      }
+      store_o_row<HD>(tO, l_run, p.o + ((long long)jb * p.Lq + q) * d + head * HD, q < p.Lq);
       // O is read before this warp's next arrival on p_full, which the next PV (that
       // overwrites O) waits for: tmem_ld32 waits for its loads to complete
     }

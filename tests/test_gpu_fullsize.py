@@ -161,13 +161,15 @@ def test_full_size_fused_cache_step_every_element(B):
         np.testing.assert_allclose(st["delta"][i].cpu().numpy(), v[i] - x[i], rtol=1e-6, atol=1e-6)
 
 
-def test_composed_block_and_head_full_length_sampled_rows(B):
+@pytest.mark.parametrize("base", ["wan1.3b", "wan1.3b-short"])
+def test_composed_block_and_head_full_length_sampled_rows(B, base):
     """The composed DiT forward (patch embed, LayerNorm + adaLN, QKV scatter, self-attention
-    over all 32760 tokens, gated O projection, cross-attention to the 512 text tokens, GELU
-    FFN, head) of one 1.3B-width block on a compacted subset of 4 candidates (idx 0, 2, 3),
-    against the oracle's one-block velocity on 40 sampled token rows x all 64 features;
-    full-length K/V on both sides.  The row outside the subset stays untouched."""
-    m = synth.replace_model(synth.WAN_1_3B, blocks=1)
+    over all tokens -- 32760 for the best-of-4 and beam latent, 14040 for the short clips --,
+    gated O projection, cross-attention to the 512 text tokens, GELU FFN, head) of one
+    1.3B-width block on a compacted subset of 4 candidates (idx 0, 2, 3), against the
+    oracle's one-block velocity on 40 sampled token rows x all 64 features; full-length K/V
+    on both sides.  The row outside the subset stays untouched."""
+    m = synth.replace_model(synth.WAN_1_3B if base == "wan1.3b" else synth.WAN_1_3B_SHORT, blocks=1)
     flat, params = synth.make_params(m)
     ctx = synth.text_context(m)
     x1 = synth.initial_noise(m, range(NC))
