@@ -209,10 +209,10 @@ cs_status cs_search_step_cfg(cs_model* model, float* x_dev, float* x_ref_dev, fl
  * Eq. skip + Eq. euler to the skipped ones (writing their score partials if target_dev
  * is given), so that a skipped candidate's x_ref and Delta are read once, x read while
  * still in L2 and written once.  Two launches and no grid-wide wait: the drift pass,
- * in which the CTA that completes a candidate's last chunk decides it, then the skip
+ * in which the CTA that arrives last on one counter takes every decision, then the skip
  * update, scheduled by programmatic dependent launch while the first drains.  Needs
  * D % 8 == 0, 32-byte aligned tensors and cs_cache_workspace_bytes(N, D) of workspace
- * (its arrival counters are cleared by the call).  cs_cache_apply_computed then updates
+ * (its arrival counter is cleared by the call).  cs_cache_apply_computed then updates
  * only the computed candidates (Eq. delta + Eq. euler, v_dev from the DiT) and, with
  * target_dev, finalises the scores of all candidates. */
 cs_status cs_cache_decide_skip(float* x_dev, const float* x_ref_dev, const float* delta_dev, float* accum_dev,
