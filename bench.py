@@ -5,6 +5,8 @@ N candidates, the DiT forward of the computing subset (30 blocks at the Wan2.1-1
 shape), the fused Delta/Euler update, and (on the last step of a rollout) scoring and
 top-k.  Warm-up steps run on a throwaway search; the timed steps run a fresh search
 from step 1 (a new search starts after T steps).  Metric: candidate-denoising-steps/s.
+A second timed region then runs one complete search, steps 1..T, whatever K is, and
+reports it under `full_search` with its own per-class kernel times and clocks.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--tau T]
   python bench.py --impl reference ...   # the fp64 CPU oracle on a bounded sample
@@ -62,6 +64,13 @@ def kernel_counters(cls, path=COUNTERS):
     return None
 
 
+def measured_peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except OSError:
+        return {}
+
+
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -79,6 +88,8 @@ def parse():
                          "schedule with the skip count the paper reports (26 of 50 steps skipped)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-full-search", action="store_true",
+                    help="skip the second timed region: one complete T-step search from step 1")
     return ap.parse_args()
 
 
@@ -388,6 +399,39 @@ def run_ours(args, cfg):
     ms = max_over_ranks(ms_local, world)
     value = job_throughput(advanced, ms_local / 1e3, world)
 
+    # a second timed region: one complete search, steps 1..T (the K timed steps above cover
+    # steps 1..K of it), with the same per-class kernel timing
+    full = None
+    if not args.no_full_search:
+        model.reset_kernel_stats()
+        model.set_profiling(True)
+        f_computed = f_advanced = 0
+        barrier(world)
+        torch.cuda.synchronize()
+        with ClockSampler(local) as f_clk:
+            fe0, fe1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            fe0.record()
+            for i in range(T):
+                c, a = step(i)
+                f_computed += c
+                f_advanced += a
+            fe1.record()
+            torch.cuda.synchronize()
+            barrier(world)
+        f_ms_local = fe0.elapsed_time(fe1)
+        model.set_profiling(False)
+        f_stats = {c: model.kernel_stats(c) for c in range(5)}
+        fn_sa, fms_sa, ffl_sa = f_stats[B.KC_SELF_ATTN]
+        fn_c, fms_c, fby_c = f_stats[B.KC_CACHE]
+        f_hbm = measured_peaks().get("hbm_gbs") or 6800.0
+        f_gbs = fby_c / (fms_c / 1e3) / 1e9 if fms_c else 0.0
+        full = {"T": T, "value": job_throughput(f_advanced, f_ms_local / 1e3, world), "unit": UNIT,
+                "ms": max_over_ranks(f_ms_local, world),
+                "computed_fraction": f_computed / ((2 if mode == "cfg" else 1) * f_advanced),
+                "self_attention_tflops": (ffl_sa / (fms_sa / 1e3) / 1e12) if fms_sa else None,
+                "cache_update": {"launches": fn_c, "ms": fms_c, "gbs": f_gbs, "frac_hbm": f_gbs / f_hbm},
+                "clocks": f_clk.summary()}
+
     # end to end through the host-buffer entry point (pinned host latents in, latents + mask out)
     e2e = None
     tgrid = S.time_grid(T)
@@ -413,11 +457,7 @@ def run_ours(args, cfg):
 
     if rank != 0:
         return
-    peaks = {}
-    try:
-        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
-    except OSError:
-        pass
+    peaks = measured_peaks()
     n_sa, ms_sa, fl_sa = stats[B.KC_SELF_ATTN]
     peak_tf = peaks.get("bf16_tflops_sustained")
     peak_src = "measured (sustained)" if peak_tf else "fallback (sustained)"
@@ -467,6 +507,8 @@ def run_ours(args, cfg):
         "gpu_launches": launches,
         "clocks": clocks,
     }
+    if full:
+        line["full_search"] = full
     if e2e:
         line["e2e"] = e2e
     if not args.no_cpu_baseline and world == 1:

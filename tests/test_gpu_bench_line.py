@@ -1,0 +1,32 @@
+"""The bench's own arm on the GPU (tiny workload, a few steps): one JSON line with the
+contract's keys, the kernel launches counted, the end-to-end number through the host-buffer
+entry point, and the second timed region that runs one complete search."""
+import json
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.mark.gpu
+def test_bench_line_on_the_tiny_workload():
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--config", "tiny", "--steps", "4",
+                        "--warmup", "3", "--no-cpu-baseline"], capture_output=True, text=True, timeout=900, cwd=ROOT)
+    assert r.returncode == 0, r.stderr[-3000:]
+    lines = [ln for ln in r.stdout.strip().splitlines() if ln.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better",
+                "scaling", "vs_baseline", "dtype", "data", "config", "roofline", "e2e", "gpu_launches", "clocks",
+                "kernels", "full_search"):
+        assert key in d, key
+    assert d["steps"] == 4 and d["warmup"] == 3 and d["n_gpus"] == 1 and d["value"] > 0
+    assert d["gpu_launches"] > 0 and d["config"]["workload"] == "tiny"
+    assert d["roofline"]["bound"] == "tensor" and d["roofline"]["achieved"] > 0
+    assert d["e2e"]["value"] > 0 and d["e2e"]["h2d_bytes_per_step"] > 0 and d["e2e"]["d2h_bytes_per_step"] > 0
+    f = d["full_search"]
+    assert f["T"] == d["config"]["T"] and f["value"] > 0 and 0 < f["computed_fraction"] <= 1
+    assert f["cache_update"]["launches"] > 0 and f["unit"] == d["unit"]
