@@ -6,7 +6,9 @@ shape), the fused Delta/Euler update, and (on the last step of a rollout) scorin
 top-k.  Warm-up steps run on a throwaway search; the timed steps run a fresh search
 from step 1 (a new search starts after T steps).  Metric: candidate-denoising-steps/s.
 A second timed region then runs one complete search, steps 1..T, whatever K is, and
-reports it under `full_search` with its own per-class kernel times and clocks.
+reports it under `full_search` with its own per-class kernel times and clocks.  The cache
+step is also timed alone on large batches (`cache_alone`: 16 candidates of the 1.3B latent,
+32 of the short clip, and the bench's own N), single calls after an L2-evicting write.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--tau T]
   python bench.py --impl reference ...   # the fp64 CPU oracle on a bounded sample
@@ -90,6 +92,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-full-search", action="store_true",
                     help="skip the second timed region: one complete T-step search from step 1")
+    ap.add_argument("--no-cache-alone", action="store_true",
+                    help="skip the cache step timed alone on large batches (N 16 and 32, and the bench's N)")
     return ap.parse_args()
 
 
@@ -432,6 +436,24 @@ def run_ours(args, cfg):
                 "cache_update": {"launches": fn_c, "ms": fms_c, "gbs": f_gbs, "frac_hbm": f_gbs / f_hbm},
                 "clocks": f_clk.summary()}
 
+    # the cache step alone on large batches (16 candidates of the 1.3B latent, 32 of the short
+    # clip) and at the bench's own N: one free step's decide + skip and computed update per call
+    cache_alone = None
+    if not args.no_cache_alone and rank == 0:
+        from paper_2607_23159_gb300 import kernel_bench as KB
+        hbm = measured_peaks().get("hbm_gbs") or 6800.0
+        cases = []
+        for n_c, lat, sf in ((16, (16, 21, 60, 104), 1.0), (16, (16, 21, 60, 104), 0.5), (32, (16, 9, 30, 52), 1.0),
+                             (32, (16, 9, 30, 52), 0.5), (N, (m.C, m.F, m.H, m.W), 1.0), (N, (m.C, m.F, m.H, m.W), 0.5)):
+            c_ms, c_bytes, c_skip = KB.cache_step(n_c, lat, sf)
+            gbs = c_bytes / (c_ms / 1e3) / 1e9
+            cases.append({"N": n_c, "latent": "x".join(map(str, lat)), "skipped": c_skip, "us": c_ms * 1e3,
+                          "gbs": gbs, "frac_hbm": gbs / hbm})
+        torch.cuda.empty_cache()
+        cache_alone = {"what": "cs_cache_decide_skip + cs_cache_apply_tokens on one free step; median of 9 "
+                               "single calls, each after a 256 MB L2-evicting write; 16 D bytes per skipped "
+                               "candidate, 24 D per computed one", "cases": cases}
+
     # end to end through the host-buffer entry point (pinned host latents in, latents + mask out)
     e2e = None
     tgrid = S.time_grid(T)
@@ -509,6 +531,8 @@ def run_ours(args, cfg):
     }
     if full:
         line["full_search"] = full
+    if cache_alone:
+        line["cache_alone"] = cache_alone
     if e2e:
         line["e2e"] = e2e
     if not args.no_cpu_baseline and world == 1:

@@ -53,6 +53,44 @@ def _time_cold(fn, reps, warmup):
     return times[len(times) // 2]
 
 
+def cache_step(N, lat, skip_frac, reps=9, warmup=3, seed=0):
+    """One free step's cache work for N candidates on a C x F x H x W latent, as the search
+    step runs it: cs_cache_decide_skip (drift, decision, skipped updates), then
+    cs_cache_apply_tokens for the computing candidates (head output in token layout).  The
+    round(N (1 - skip_frac)) candidates that compute are a seeded random subset.  Returns
+    (median ms of single calls after an L2-evicting write, algorithmic bytes, skipped):
+    16 D bytes per skipped candidate, 24 D per computed one."""
+    import torch
+    from paper_2607_23159_gb300 import binding as B
+    dev = "cuda"
+    C_, F_, H_, W_ = lat
+    D = C_ * F_ * H_ * W_
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+    st = B.new_state(N, D)
+    st["x"].normal_(generator=g)
+    st["x_ref"].copy_(st["x"] * 0.99)
+    st["delta"].normal_(generator=g)
+    st["has_ref"].fill_(1)
+    ws = torch.zeros(B.cache_workspace_bytes(N, D) // 4 + 1, device=dev)
+    skip = torch.zeros(N, dtype=torch.uint8, device=dev)
+    idx = torch.zeros(N, dtype=torch.int32, device=dev)
+    nc = torch.zeros(1, dtype=torch.int32, device=dev)
+    n_comp = int(round(N * (1.0 - skip_frac)))
+    force = torch.zeros(N, dtype=torch.uint8, device=dev)
+    force[torch.randperm(N, generator=g, device=dev)[:n_comp]] = 1
+    hout = torch.randn(max(1, n_comp) * F_ * (H_ // 2) * (W_ // 2), 4 * C_, device=dev, generator=g)
+    comp_idx = torch.nonzero(force).to(torch.int32).reshape(-1)
+
+    def run():
+        B.cache_decide_skip(st["x"], st["x_ref"], st["delta"], st["accum"], st["has_ref"], 20, 50, 0.6, 0.58,
+                            0.1, 5, 5, skip, idx, nc, ws, force=force)
+        B.cache_apply_tokens(st, skip, hout, comp_idx, n_comp, C_, F_, H_, W_, 0.6, 0.58)
+    ms = _time_cold(run, reps, warmup)
+    n_skip = N - n_comp
+    return ms, (n_skip * 16.0 + n_comp * 24.0) * D, n_skip
+
+
 def main():
     import torch
     from paper_2607_23159_gb300 import build
@@ -158,7 +196,11 @@ def main():
         N, D = a.N, a.D
         lat = [int(v) for v in a.latent.split("x")]
         if a.kernel == "cache-tokens":
+            ms, byts, n_skip = cache_step(N, lat, a.skip_frac, a.reps, a.warmup)
             D = lat[0] * lat[1] * lat[2] * lat[3]
+            out.update(shape=dict(N=N, D=D, skipped=n_skip), ms=ms, gbs=byts / (ms / 1e3) / 1e9)
+            print(json.dumps(out), flush=True)
+            return
         st = B.new_state(N, D)
         st["x"].normal_()
         st["x_ref"].copy_(st["x"] * 0.99)
@@ -170,17 +212,9 @@ def main():
         idx = torch.zeros(N, dtype=torch.int32, device=dev)
         nc = torch.zeros(1, dtype=torch.int32, device=dev)
         force = (torch.rand(N, device=dev) >= a.skip_frac).to(torch.uint8)
-        n_comp = int(force.sum())
-        C_, F_, H_, W_ = lat
-        hout = torch.randn(max(1, n_comp) * F_ * (H_ // 2) * (W_ // 2), 4 * C_, device=dev)
-        comp_idx = torch.nonzero(force).to(torch.int32).reshape(-1)
 
         def run():
-            if a.kernel == "cache-tokens":   # the search step's pair: decide + skip, then the computed update
-                B.cache_decide_skip(st["x"], st["x_ref"], st["delta"], st["accum"], st["has_ref"], 20, 50, 0.6, 0.58,
-                                    0.1, 5, 5, skip, idx, nc, ws, force=force)
-                B.cache_apply_tokens(st, skip, hout, comp_idx, n_comp, C_, F_, H_, W_, 0.6, 0.58)
-            elif a.kernel == "cache-fused":
+            if a.kernel == "cache-fused":
                 B.cache_decide_skip(st["x"], st["x_ref"], st["delta"], st["accum"], st["has_ref"], 20, 50, 0.6, 0.58,
                                     0.1, 5, 5, skip, idx, nc, ws, force=force)
                 B.cache_apply_computed(st["x"], st["x_ref"], st["delta"], v, skip, 0.6, 0.58)
