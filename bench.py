@@ -243,7 +243,7 @@ def cpu_cores():
         return os.cpu_count() or 1
 
 
-def cpu_baseline(cfg, rows=512):
+def cpu_baseline(cfg, rows=2048):
     s_per_cs, sample_s = oracle_sample_seconds(cfg.model, rows=rows)
     rows = min(rows, cfg.model.L)
     return {"value": 1.0 / s_per_cs, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",

@@ -199,7 +199,8 @@ def _velocity_np(x, k):
     return a * x + b
 
 
-@pytest.mark.parametrize("N,D,tau,K_w,K_c", [(5, 4096, 0.08, 1, 1), (3, 1001, 0.15, 0, 0), (4, 70000, 0.0, 1, 1)])
+@pytest.mark.parametrize("N,D,tau,K_w,K_c", [(5, 4096, 0.08, 1, 1), (3, 1001, 0.15, 0, 0), (4, 70000, 0.0, 1, 1),
+                                             (4096, 24, 0.1, 1, 1)])   # the most candidates a call takes
 def test_cache_rule_matches_oracle(B, N, D, tau, K_w, K_c):
     T = 8
     t = O.time_grid(T)
@@ -304,7 +305,9 @@ def test_score_topk_and_beam_refill(B):
     np.testing.assert_array_equal(dst["accum"].cpu().numpy(), np.array([s.a for s in ns], np.float32))
 
 
-@pytest.mark.parametrize("N,D,score", [(4, 2096640, True), (7, 50000, False), (16, 8192 * 3, True)])
+@pytest.mark.parametrize("N,D,score", [(4, 2096640, True), (7, 50000, False), (16, 8192 * 3, True),
+                                     (2, 8192 + 8, False),      # one full chunk and an 8-element tail
+                                     (4096, 16, True)])         # the most candidates a call takes
 def test_fused_decide_skip_equals_two_pass_path(B, N, D, score):
     """cs_cache_decide_skip + cs_cache_apply_computed give the same state bits as
     cs_cache_decide + cs_cache_apply, over three steps (forced, free, scored)."""
