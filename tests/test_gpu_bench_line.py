@@ -33,3 +33,25 @@ def test_bench_line_on_the_tiny_workload():
     cases = d["cache_alone"]["cases"]
     assert [(c["N"], c["latent"]) for c in cases[:4]] == [(16, "16x21x60x104")] * 2 + [(32, "16x9x30x52")] * 2
     assert all(c["gbs"] > 0 and 0 <= c["skipped"] <= c["N"] for c in cases)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("extra", [["--search", "pruned"], ["--search", "static"], ["--search", "commit"],
+                                   ["--search", "cfg"], ["--mask", "paper-density"], ["--tau", "0"]])
+def test_bench_search_modes_on_the_tiny_workload(extra):
+    """Every search mode the bench can time runs through its own arm and prints one line."""
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--config", "tiny", "--steps", "10",
+                        "--warmup", "3", "--no-cpu-baseline", "--no-cache-alone", *extra],
+                       capture_output=True, text=True, timeout=900, cwd=ROOT)
+    assert r.returncode == 0, r.stderr[-3000:]
+    lines = [ln for ln in r.stdout.strip().splitlines() if ln.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["value"] > 0 and d["gpu_launches"] > 0 and 0 < d["computed_fraction"] <= 1
+    assert d["full_search"]["value"] > 0
+    if "--search" in extra:
+        assert d["config"]["search"] == extra[1]
+    if extra == ["--search", "commit"]:
+        assert d["config"]["N"] == 1 and d["computed_fraction"] == 1.0
+    if extra == ["--tau", "0"]:
+        assert d["computed_fraction"] == 1.0
