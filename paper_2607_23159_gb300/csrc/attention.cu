@@ -626,7 +626,7 @@ __global__ void __launch_bounds__(AttnCfg<HD>::THREADS, 1)
   attn_body<HD>(tmQ, tmK, tmV, p);
 }
 
-constexpr int kPersistMaxKeys = 2048;
+constexpr int kPersistMaxKeys = 8192;
 
 template <int HD>
 static cs_status launch_attn(const void* q, const void* k, const void* vt, void* o, int B, int heads, int Lq, int Lk,
@@ -661,10 +661,12 @@ static cs_status launch_attn(const void* q, const void* k, const void* vt, void*
   a.err = err;
   dim3 grid((Lq + 255) / 256, BH);
   if (Lk <= kPersistMaxKeys) {
-    // short key loops (cross-attention over the text): one CTA per SM walks the items, so
-    // that an item's Q load, first scores and O epilogue overlap its neighbours' work
-    // (measured at 4 x 12 x 32760 x 512: 973 -> 1026 TFLOP/s; at 32760 keys the same
-    // form measured 1-3 % slower than one item per CTA, so long key loops keep that)
+    // short key loops (cross-attention over the text, short clips): one CTA per SM walks the
+    // items, so that an item's Q load, first scores and O epilogue overlap its neighbours'
+    // work.  Measured (same bits either way): 4 x 12 x 32760 x 512 973 -> 1026 TFLOP/s,
+    // 8 x 12 x 4096^2 1370-1416 -> 1476, 4 x 12 x 8192^2 1495-1523 -> 1548; at 14040 keys
+    // +2 % at 4 batch items and -1 % at 32, at 32760 keys -0.5 %, so longer loops keep
+    // one item per CTA
     auto kern = attn_tcgen05_persist_kernel<HD>;
     CS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
     const int items = grid.x * grid.y;

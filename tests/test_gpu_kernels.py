@@ -144,11 +144,12 @@ def _attn_case(B, hd, heads, nb, Lq, Lk, kv_shared, qscale, seed, kramp=0.0):
     (128, 2, 2, 300, 200, False, 1.0),     # ragged queries and keys, 2 key tiles
     (128, 1, 1, 257, 1000, False, 3.0),    # peaked softmax: running max changes, lazy rescale
     (128, 3, 2, 130, 512, True, 1.0),      # cross-attention: K/V shared by all batch items
+    (128, 2, 2, 520, 3000, False, 2.0),    # persistent form on a longer key loop (3 items per batch item)
     (32, 4, 4, 48, 48, False, 1.0),        # tiny model shape (one partial tile)
     (32, 4, 2, 48, 16, True, 2.0),         # tiny cross-attention, 16 text tokens
     (128, 2, 1, 1, 129, False, 1.0),       # one query row; the last key tile holds one key
     (128, 2, 2, 256, 1, False, 1.0),       # a single key: one tile, one valid column
-    (128, 1, 2, 300, 2100, False, 1.0),    # more than 2048 keys: per-thread output stores, ragged rows
+    (128, 1, 2, 300, 8300, False, 1.0),    # more than 8192 keys: one item per CTA, ragged rows and keys
 ])
 def test_attention_matches_oracle(B, hd, heads, nb, Lq, Lk, kv_shared, qscale):
     q, k, v, got = _attn_case(B, hd, heads, nb, Lq, Lk, kv_shared, qscale, seed=hd + Lq + Lk)
