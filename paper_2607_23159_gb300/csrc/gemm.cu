@@ -88,12 +88,13 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& p, int m, int n, 
   for (int j = 0; j < 32; ++j) f[j] = __uint_as_float(r[j]);
   const bool full = (n + 32 <= p.N);
   if (p.bias) {
-    if (full) {
+    if (full) {   // packed f32x2 adds (the same bits as scalar ones)
       const float4* b4 = reinterpret_cast<const float4*>(p.bias + n);
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
         const float4 b = __ldg(b4 + j);
-        f[4 * j] += b.x; f[4 * j + 1] += b.y; f[4 * j + 2] += b.z; f[4 * j + 3] += b.w;
+        f2_unpack(f2_add(f2_pack(f[4 * j], f[4 * j + 1]), f2_pack(b.x, b.y)), f[4 * j], f[4 * j + 1]);
+        f2_unpack(f2_add(f2_pack(f[4 * j + 2], f[4 * j + 3]), f2_pack(b.z, b.w)), f[4 * j + 2], f[4 * j + 3]);
       }
     } else {
       for (int j = 0; j < 32; ++j)
@@ -350,10 +351,12 @@ __global__ void __launch_bounds__(192, 1)
               float v[8];
 #pragma unroll
               for (int j = 0; j < 8; ++j) v[j] = __uint_as_float(u < 4 ? r0[8 * u + j] : r1[8 * (u - 4) + j]);
-              if (b4) {
+              if (b4) {   // packed f32x2 adds: the same bits, half the instructions beside the main loop
                 const float4 ba = __ldg(b4 + 2 * u), bb = __ldg(b4 + 2 * u + 1);
-                v[0] += ba.x; v[1] += ba.y; v[2] += ba.z; v[3] += ba.w;
-                v[4] += bb.x; v[5] += bb.y; v[6] += bb.z; v[7] += bb.w;
+                f2_unpack(f2_add(f2_pack(v[0], v[1]), f2_pack(ba.x, ba.y)), v[0], v[1]);
+                f2_unpack(f2_add(f2_pack(v[2], v[3]), f2_pack(ba.z, ba.w)), v[2], v[3]);
+                f2_unpack(f2_add(f2_pack(v[4], v[5]), f2_pack(bb.x, bb.y)), v[4], v[5]);
+                f2_unpack(f2_add(f2_pack(v[6], v[7]), f2_pack(bb.z, bb.w)), v[6], v[7]);
               }
               if constexpr (EPI == CS_EPI_GELU_BF16) {
 #pragma unroll
@@ -407,15 +410,20 @@ __global__ void __launch_bounds__(192, 1)
                                                                    : nullptr;
 #pragma unroll
             for (int u = 0; u < 8; ++u) {
-              float4 v = make_float4(f[4 * u], f[4 * u + 1], f[4 * u + 2], f[4 * u + 3]);
-              if (b4) {
+              float4 v;
+              uint64_t lo = f2_pack(f[4 * u], f[4 * u + 1]), hi = f2_pack(f[4 * u + 2], f[4 * u + 3]);
+              if (b4) {   // packed f32x2 add and multiply: the same bits as scalar ones
                 const float4 b = __ldg(b4 + u);
-                v.x += b.x; v.y += b.y; v.z += b.z; v.w += b.w;
+                lo = f2_add(lo, f2_pack(b.x, b.y));
+                hi = f2_add(hi, f2_pack(b.z, b.w));
               }
               if (g4) {
                 const float4 g = __ldg(g4 + u);
-                v.x *= g.x; v.y *= g.y; v.z *= g.z; v.w *= g.w;
+                lo = f2_mul(lo, f2_pack(g.x, g.y));
+                hi = f2_mul(hi, f2_pack(g.z, g.w));
               }
+              f2_unpack(lo, v.x, v.y);
+              f2_unpack(hi, v.z, v.w);
               *reinterpret_cast<float4*>(buf + lane * 128 + ((u ^ (lane & 7)) << 4)) = v;
             }
             fence_proxy_async_smem();
