@@ -25,6 +25,8 @@ def test_reference_arm_prints_one_contract_line():
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    # the measured time of a sample step, and the whole-step time the value is scaled from
+    assert 0 < d["ms_per_step"] < 600e3 and d["ms_per_full_step_extrapolated"] > 0
 
 
 def test_clock_summary_parses_nvidia_smi_samples():
