@@ -59,6 +59,10 @@ def test_committed_kernel_counters_parse_and_track_their_source(tmp_path):
     rec = bench.kernel_counters("self_attention")
     assert rec is not None and rec["units"] > 0 and rec["dram_bytes"] > 0 and 0 < rec["tensor_active"] <= 100
     assert os.path.exists(os.path.join(ROOT, "profiles", rec["summary"]))
+    # every committed capture was taken on the kernel sources as they are now
+    for cls in ("self_attention", "cross_attention", "gemm", "gemm_ffn_down"):
+        r = bench.kernel_counters(cls)
+        assert r is not None and r["stale"] is False, cls
     fake = tmp_path / "c.txt"
     fake.write_text("# comment\nclass=self_attention kernel=k units=2 dram_bytes=1e6 tensor_active=50 sm_mhz=1900 "
                     "src=attention.cu:0000000000000000 summary=x.md\n")
