@@ -39,6 +39,7 @@ struct GemmArgs {
   __nv_bfloat16* vt;
   int L, d, heads, hd, hd_s, Lv, which_base;
   int tma_out;   // float32 epilogues: stage in shared memory and TMA-store / TMA-reduce-add the output
+  int tma_qk;    // attention-layout epilogue: Q and K rows staged and TMA-stored (tmC = Q, tmD = K)
   int* err;
 };
 
@@ -174,7 +175,8 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& p, int m, int n, 
 template <int BN, int EPI, int MODE>
 __global__ void __launch_bounds__(192, 1)
     gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                        const __grid_constant__ CUtensorMap tmC, const GemmArgs p) {
+                        const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmD,
+                        const GemmArgs p) {
   using Cfg = GemmCfg<BN, MODE>;
   static_assert(MODE == 0 || MODE == 2, "MODE 0 (one CTA per tile) or 2 (two-SM MMA)");
   constexpr bool TWO_SM = MODE == 2;   // one cta_group::2 MMA stream issued by the cluster's rank 0
@@ -324,7 +326,8 @@ __global__ void __launch_bounds__(192, 1)
     int acc = 0;
     uint32_t acc_phase = 0;
     int nout = 0;   // chunks this warp has handed to TMA
-    if (lane == 0 && p.tma_out) tma_prefetch_desc(&tmC);
+    if (lane == 0 && (p.tma_out || p.tma_qk)) tma_prefetch_desc(&tmC);
+    if (lane == 0 && p.tma_qk) tma_prefetch_desc(&tmD);
     for (int it = first; it < items; it += stride) {
       if (!__all_sync(0xffffffffu, mbar_wait(&tfull[acc], acc_phase, abort_flag, p.err))) break;
       tc_fence_after();
@@ -373,6 +376,72 @@ __global__ void __launch_bounds__(192, 1)
             __syncwarp();
             if (lane == 0) {
               tma_store_2d(&tmC, buf, n, m0 + sp * 32);
+              bulk_commit();
+            }
+            ++nout;
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) {
+            if (TWO_SM) mbar_arrive_cluster(cluster_map(&tempty[acc], 0));
+            else mbar_arrive(&tempty[acc]);
+          }
+          acc ^= 1;
+          if (acc == 0) acc_phase ^= 1;
+          continue;
+        }
+      }
+      if constexpr (EPI == CS_EPI_QKV) {
+        if (p.tma_qk) {
+          // 64 columns (one head of Q or K) at a time: a warp whose 32 rows lie in one batch item
+          // stages them and TMA-stores 32 consecutive (head, token) rows; V^T, rows that cross a
+          // batch item or pass M go through the per-thread stores
+#pragma unroll 1
+          for (int c = 0; c < BN / 64; ++c) {
+            const int n = n0 + c * 64;
+            if (n >= p.N) break;   // uniform across the warp
+            uint32_t r0[32], r1[32];
+            tmem_ld32(tbase + c * 64, r0);
+            tmem_ld32(tbase + c * 64 + 32, r1);
+            const int w = p.which_base + n / p.d;
+            const int mf = m0 + sp * 32;
+            const int jb = mf / p.L;
+            const bool staged = w < 2 && mf + 31 < p.M && (mf + 31) / p.L == jb;   // uniform across the warp
+            if (!staged) {
+              if (m < p.M) {
+                epilogue_chunk<EPI>(p, m, n, r0);
+                epilogue_chunk<EPI>(p, m, n + 32, r1);
+              }
+              continue;
+            }
+            const int c0 = n % p.d, head = c0 / p.hd, e = c0 % p.hd;
+            uint8_t* buf = sOut + (sp * 2 + (nout & 1)) * 4096;
+            if (lane == 0 && nout >= 2) bulk_wait_read_1();
+            __syncwarp();
+            const float4* b4 = p.bias ? reinterpret_cast<const float4*>(p.bias + n) : nullptr;
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+              float v[8];
+#pragma unroll
+              for (int j = 0; j < 8; ++j) v[j] = __uint_as_float(u < 4 ? r0[8 * u + j] : r1[8 * (u - 4) + j]);
+              if (b4) {
+                const float4 ba = __ldg(b4 + 2 * u), bb = __ldg(b4 + 2 * u + 1);
+                f2_unpack(f2_add(f2_pack(v[0], v[1]), f2_pack(ba.x, ba.y)), v[0], v[1]);
+                f2_unpack(f2_add(f2_pack(v[2], v[3]), f2_pack(ba.z, ba.w)), v[2], v[3]);
+                f2_unpack(f2_add(f2_pack(v[4], v[5]), f2_pack(bb.x, bb.y)), v[4], v[5]);
+                f2_unpack(f2_add(f2_pack(v[6], v[7]), f2_pack(bb.z, bb.w)), v[6], v[7]);
+              }
+              uint4 wv;
+              wv.x = pack_bf16x2(v[0], v[1]);
+              wv.y = pack_bf16x2(v[2], v[3]);
+              wv.z = pack_bf16x2(v[4], v[5]);
+              wv.w = pack_bf16x2(v[6], v[7]);
+              *reinterpret_cast<uint4*>(buf + lane * 128 + ((u ^ (lane & 7)) << 4)) = wv;
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(w == 0 ? &tmC : &tmD, buf, e, (jb * p.heads + head) * p.L + (mf - jb * p.L));
               bulk_commit();
             }
             ++nout;
@@ -493,13 +562,27 @@ static cs_status launch_gemm(const void* A, const void* B, const GemmArgs& args,
     CS_TRY(make_tmap(&tc, args.out, 2, dc, sc, bc, false));
     a.tma_out = 1;
   }
+  CUtensorMap td = tc;   // unused unless a.tma_qk
+  a.tma_qk = 0;
+  if (EPI == CS_EPI_QKV && args.hd % 64 == 0 && args.d % 64 == 0 && args.N % 64 == 0 && args.q &&
+      (reinterpret_cast<uintptr_t>(args.q) & 15) == 0 && (!args.k || (reinterpret_cast<uintptr_t>(args.k) & 15) == 0)) {
+    // Q and K as 2-D [rows = (batch item, head, token), hd_s] bf16: a warp's 32 rows of one head
+    // and one batch item are 32 consecutive rows there
+    const uint64_t dq[2] = {(uint64_t)args.hd_s, (uint64_t)args.M * (uint64_t)args.heads};
+    const uint64_t sq[1] = {(uint64_t)args.hd_s * 2};
+    const uint32_t bq[2] = {64, 32};
+    CS_TRY(make_tmap(&tc, args.q, 2, dq, sq, bq, false));
+    td = tc;
+    if (args.k) CS_TRY(make_tmap(&td, args.k, 2, dq, sq, bq, false));
+    a.tma_qk = 1;
+  }
   auto kern = gemm_tcgen05_kernel<BN, EPI, MODE>;
   CS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM));
   const int m_tiles = (args.M + 127) / 128, n_tiles = (args.N + BN - 1) / BN;
   if (!PAIR) {
     const int tiles = m_tiles * n_tiles;
     const int grid = tiles < num_sms() ? tiles : num_sms();
-    kern<<<grid, 192, Cfg::SMEM, stream>>>(ta, tb, tc, a);
+    kern<<<grid, 192, Cfg::SMEM, stream>>>(ta, tb, tc, td, a);
     CS_LAUNCHED();
     return CS_OK;
   }
@@ -527,7 +610,7 @@ static cs_status launch_gemm(const void* A, const void* B, const GemmArgs& args,
   if (max_clusters == 0) return launch_gemm<BN, EPI, 0>(A, B, args, stream);   // no cluster fits: one CTA per tile
   const int items = ((m_tiles + 1) / 2) * n_tiles;
   cfg.gridDim = dim3(2 * (items < max_clusters ? items : max_clusters));
-  CS_CUDA(cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, a));
+  CS_CUDA(cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, td, a));
   CS_LAUNCHED();
   return CS_OK;
 }
