@@ -456,9 +456,10 @@ def run_ours(args, cfg):
             cases.append({"N": n_c, "latent": "x".join(map(str, lat)), "skipped": c_skip, "us": c_ms * 1e3,
                           "gbs": gbs, "frac_hbm": gbs / hbm})
         torch.cuda.empty_cache()
-        cache_alone = {"what": "cs_cache_decide_skip + cs_cache_apply_tokens on one free step; median of 9 "
-                               "single calls, each after a 256 MB L2-evicting write; 16 D bytes per skipped "
-                               "candidate, 24 D per computed one", "cases": cases}
+        cache_alone = {"what": "cs_cache_decide_skip_carry + cs_cache_apply_tokens_carry (the step's form: the "
+                               "drift carried from the previous step) on one free step; median of 9 single calls, "
+                               "each after a 256 MB L2-evicting write; 16 D bytes per skipped candidate, 20 D per "
+                               "computed one", "cases": cases}
 
     # end to end through the host-buffer entry point (pinned host latents in, latents + mask out)
     e2e = None

@@ -243,6 +243,44 @@ cs_status cs_cache_apply_tokens(float* x_dev, float* x_ref_dev, float* delta_dev
                                 float t_cur, float t_next, const float* target_dev, float* scores_dev,
                                 void* workspace_dev, float* tile_partials_dev, int* err_dev, cudaStream_t stream);
 
+/* Carried form of the two calls above (Sec. 3.1, Eq. indicator, Eq. skip, Eq. euler), the
+ * one cs_search_step runs.  The drift of step k needs ||x - x_ref|| and ||x_ref|| of the
+ * latent a candidate holds at step k, which the update of step k - 1 writes: these calls
+ * make every update also leave those two squared norms for the next step (the "carried"
+ * drift), so that a step takes its decisions without reading x or x_ref and its skip
+ * update is the only pass over a skipped candidate's state (read x, Delta, x_ref; write
+ * x).  Results are those of cs_cache_decide_skip + cs_cache_apply_tokens except for the
+ * order in which the drift's sums are added (float32, fixed per candidate).
+ *   has_ref = 3 (bit 1 set) marks a candidate whose carried sums belong to its current
+ *   x and x_ref; the carrying calls leave 3, every other call leaves 1 (or 0).  A caller
+ *   that changes x or x_ref of a candidate between two steps in any other way must clear
+ *   bit 1 of its has_ref (has_ref &= 1).
+ *   step_ws_dev: cs_cache_step_bytes(N, C, F, H, W) bytes of device memory, zero-filled
+ *   before its first use and then kept with the state (it holds the carried sums per
+ *   candidate row, by the parity of step_k); every call leaves its counters at zero.
+ *   Use one step_ws with one N and latent shape.
+ *   carried = 1: on a free step the decisions use the sums the previous step (step_k - 1)
+ *   left.  If a cached candidate has none (has_ref == 1), the call changes nothing and
+ *   writes *n_compute_dev = -1: call again with carried = 0.  carried = 0: a drift pass
+ *   reads x and x_ref (as cs_cache_decide_skip), then the skip update runs.  Inside the
+ *   warm-up / cool-down window no drift is needed and `carried` does not matter.
+ *   Either way the skipped candidates leave their sums for step_k + 1 (has_ref = 3), and
+ *   cs_cache_apply_tokens_carry does the same for the computed ones.
+ * Latent shape and alignment as cs_cache_apply_tokens; N <= 4096.  Errors as
+ * cs_cache_decide_skip. */
+size_t cs_cache_step_bytes(int N, int C, int F, int H, int W);
+cs_status cs_cache_decide_skip_carry(float* x_dev, const float* x_ref_dev, const float* delta_dev,
+                                     float* accum_dev, uint8_t* has_ref_dev, int N, int C, int F, int H, int W,
+                                     int step_k, int T, float t_cur, float t_next, float tau, int K_w, int K_c,
+                                     const uint8_t* force_compute_dev, uint8_t* skip_mask_dev,
+                                     int32_t* compute_idx_dev, int32_t* n_compute_dev, const float* target_dev,
+                                     int carried, void* step_ws_dev, int* err_dev, cudaStream_t stream);
+cs_status cs_cache_apply_tokens_carry(float* x_dev, float* x_ref_dev, float* delta_dev, float* accum_dev,
+                                      uint8_t* has_ref_dev, uint8_t* skip_mask_dev, const float* hout_dev,
+                                      const int32_t* compute_idx_dev, int n_c, int N, int C, int F, int H, int W,
+                                      int step_k, float t_cur, float t_next, const float* target_dev,
+                                      float* scores_dev, void* step_ws_dev, int* err_dev, cudaStream_t stream);
+
 /* One denoising step of N candidates (the unit of work of the search):
  * cs_cache_decide_skip, then the DiT forward (as cs_dit_forward) on the computing
  * subset, then the computed candidates' update from the head's token output
@@ -250,6 +288,12 @@ cs_status cs_cache_apply_tokens(float* x_dev, float* x_ref_dev, float* delta_dev
  * cs_cache_apply_computed instead).
  * State buffers (x, x_ref, delta: [N][D]; accum: [N]; has_ref: [N]) are caller-owned
  * device memory and are updated in place; a fresh search starts with has_ref = 0.
+ * With the token-layout update, the step takes the carried form
+ * (cs_cache_decide_skip_carry, cs_cache_apply_tokens_carry) with the model's own step
+ * workspace: a step uses the drift sums the previous call left when that call was step
+ * k - 1 on the same state buffers and N, and otherwise (or when a candidate's has_ref is
+ * 1) runs the drift pass; writes to x or x_ref between steps other than through these
+ * calls must clear bit 1 of the candidate's has_ref, as described there.
  * Synchronises once to read the number of computing candidates; that count is returned
  * in *n_computed (host, nullable).  A warm-up or cool-down step without a forced mask
  * computes every candidate (Sec. 3.1): it takes no decision pass and does not
@@ -278,7 +322,8 @@ cs_status cs_score(const float* x_dev, const float* target_dev, int N, long long
 cs_status cs_select_topk(const float* scores_dev, int N, int k, int32_t* idx_dev, cudaStream_t stream);
 
 /* Beam refill: destination slot s = p*(1+children) + j takes the full state of
- * candidate survivors[p] (x, x_ref, delta, accum, has_ref); for j > 0 (a child) it adds
+ * candidate survivors[p] (x, x_ref, delta, accum, has_ref as 0 or 1: a carried drift
+ * belongs to the source row and is not copied); for j > 0 (a child) it adds
  * sigma * noise[p*children + j - 1] to x.  src and dst buffers must not overlap.
  * survivors_dev: int32 [keep]; noise_dev: [keep*children][D]. */
 cs_status cs_beam_refill(const float* src_x, const float* src_x_ref, const float* src_delta,

@@ -66,6 +66,10 @@ _SIGS = {
     "cs_cache_decide_skip": (I, [P, P, P, P, P, I, LL, I, I, F, F, F, I, I, P, P, P, P, P, P, P, P]),
     "cs_cache_apply_computed": (I, [P, P, P, P, P, I, LL, F, F, P, P, P, P]),
     "cs_cache_apply_tokens": (I, [P, P, P, P, P, P, P, P, I, I, I, I, I, I, F, F, P, P, P, P, P, P]),
+    "cs_cache_step_bytes": (SZ, [I, I, I, I, I]),
+    "cs_cache_decide_skip_carry": (I, [P, P, P, P, P, I, I, I, I, I, I, I, F, F, F, I, I, P, P, P, P, P, I, P, P,
+                                       P]),
+    "cs_cache_apply_tokens_carry": (I, [P, P, P, P, P, P, P, P, I, I, I, I, I, I, I, F, F, P, P, P, P, P]),
     "cs_search_step": (I, [P, P, P, P, P, P, I, I, I, F, F, F, I, I, P, P, P, P, P, P]),
     "cs_search_step_host": (I, [P, P, P, P, P, P, I, I, I, F, F, F, I, I, P, P, P]),
     "cs_score": (I, [P, P, I, LL, P, P, P]),
@@ -191,6 +195,33 @@ def cache_apply_tokens(st, skip_mask, hout, compute_idx, n_c, C, F, H, W, t_cur,
                                     _ptr(st["has_ref"]), _ptr(skip_mask), _ptr(hout), _ptr(compute_idx), n_c, N, C,
                                     F, H, W, t_cur, t_next, _ptr(target), _ptr(scores), _ptr(workspace),
                                     _ptr(tile_partials), _ptr(err), _stream(stream)))
+
+
+def cache_step_bytes(N: int, C: int, F: int, H: int, W: int) -> int:
+    return int(lib.cs_cache_step_bytes(N, C, F, H, W))
+
+
+def cache_decide_skip_carry(st, lat, step_k, T, t_cur, t_next, tau, K_w, K_c, skip_mask, compute_idx, n_compute,
+                            step_ws, carried, force=None, target=None, err=None, stream=None):
+    """cs_cache_decide_skip_carry on state dict ``st``; ``lat`` = (C, F, H, W)."""
+    N = st["x"].shape[0]
+    C_, F_, H_, W_ = lat
+    check(lib.cs_cache_decide_skip_carry(_ptr(st["x"]), _ptr(st["x_ref"]), _ptr(st["delta"]), _ptr(st["accum"]),
+                                         _ptr(st["has_ref"]), N, C_, F_, H_, W_, step_k, T, t_cur, t_next, tau, K_w,
+                                         K_c, _ptr(force), _ptr(skip_mask), _ptr(compute_idx), _ptr(n_compute),
+                                         _ptr(target), 1 if carried else 0, _ptr(step_ws), _ptr(err),
+                                         _stream(stream)))
+
+
+def cache_apply_tokens_carry(st, skip_mask, hout, compute_idx, n_c, lat, step_k, t_cur, t_next, step_ws,
+                             target=None, scores=None, err=None, stream=None):
+    """cs_cache_apply_tokens_carry: the computed update that also leaves the next step's drift."""
+    N = st["x"].shape[0]
+    C_, F_, H_, W_ = lat
+    check(lib.cs_cache_apply_tokens_carry(_ptr(st["x"]), _ptr(st["x_ref"]), _ptr(st["delta"]), _ptr(st["accum"]),
+                                          _ptr(st["has_ref"]), _ptr(skip_mask), _ptr(hout), _ptr(compute_idx), n_c,
+                                          N, C_, F_, H_, W_, step_k, t_cur, t_next, _ptr(target), _ptr(scores),
+                                          _ptr(step_ws), _ptr(err), _stream(stream)))
 
 
 def cache_apply(x, x_ref, delta, v, skip_mask, t_cur, t_next, workspace=None, target=None, scores=None,

@@ -59,6 +59,15 @@ struct cs_model {
   int32_t* cache_sidx;        // skipped candidates [max_batch] and their count
   float* tpart;       // score partials of computed candidates per token row [max_batch][F*H/2]
   bool tokens_update = false;   // computed update straight from the head's token output
+  // carried drift (token-layout update only): per candidate slot, the drift sums of the
+  // latent the last step left, and which state buffers and step they belong to
+  void* carry_ws = nullptr;
+  cs::CarryState carry{};
+  struct {
+    const void *x = nullptr, *x_ref = nullptr, *delta = nullptr, *accum = nullptr, *has_ref = nullptr;
+    int N = 0, k = 0;
+    bool valid = false;
+  } carry_tag;
   uint8_t* skip_tmp;
   void* cache_ws;
   int* err;
@@ -189,6 +198,18 @@ static cs_status warm_cache_kernels(cs_model* m) {
                                 0.5f, score ? y : nullptr, small + 1, reinterpret_cast<float*>(m->cache_ws) + 2 * ((D + 8191) / 8192),
                                 small + 8, 1, m->err, 0));
   }
+  // the carried form: the drift pass with the carrying skip update, the decision from the
+  // carried drift, and the carrying computed update (slot 0 of the model's carry state;
+  // the model's step uses a carried drift only after a step of its own wrote it)
+  for (int score = 0; score < 2; ++score) {
+    CS_CUDA(cudaMemset(has_ref, 1, 1));
+    CS_TRY(cs::carry_decide_skip_run(x, xr, dl, small, has_ref, 1, 2, 4, 1.f, 0.75f, 1e30f, 0, 0, nullptr, skip,
+                                     m->idx, m->n_compute, score ? y : nullptr, false, m->carry, m->err, 0));
+    CS_TRY(cs::carry_decide_skip_run(x, xr, dl, small, has_ref, 1, 3, 4, 0.75f, 0.5f, 1e30f, 0, 0, nullptr, skip,
+                                     m->idx, m->n_compute, score ? y : nullptr, true, m->carry, m->err, 0));
+    CS_TRY(cs::carry_apply_tokens_run(x, xr, dl, small, has_ref, skip, m->hout, m->idx_all, 1, 1, c.C, c.F, c.H, c.W,
+                                      4, 0.5f, 0.25f, score ? y : nullptr, small + 1, m->carry, 1, m->err, 0));
+  }
   CS_CUDA(cudaDeviceSynchronize());
   CS_CUDA(cudaMemset(m->err, 0, sizeof(int)));
   return CS_OK;
@@ -303,6 +324,7 @@ extern "C" cs_status cs_init_model(const cs_model_config* cfg, cs_model** out) {
   items.push_back({reinterpret_cast<void**>(&m->n_compute), 16});
   items.push_back({reinterpret_cast<void**>(&m->skip_tmp), (size_t)cfg->max_batch});
   items.push_back({&m->cache_ws, cs_cache_workspace_bytes(cfg->max_batch, m->D)});
+  items.push_back({&m->carry_ws, cs::carry_state_bytes(cfg->max_batch, m->D, cfg->F * (cfg->H / 2))});
   items.push_back({reinterpret_cast<void**>(&m->err), 16});
   items.push_back({reinterpret_cast<void**>(&m->mod_offs_dev), nb * sizeof(float*)});
   total = 0;
@@ -325,6 +347,7 @@ extern "C" cs_status cs_init_model(const cs_model_config* cfg, cs_model** out) {
   for (int i = 0; i < cfg->max_batch; ++i) iota[i] = i;
   cudaMemcpy(m->idx_all, iota.data(), iota.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
   m->tokens_update = cs::apply_tokens_supported(cfg->C, cfg->F, cfg->H, cfg->W);
+  m->carry = cs::CarryState{m->carry_ws, cfg->max_batch, m->D, cfg->F * (cfg->H / 2)};
   if (cs::load_cache_kernels() != CS_OK || warm_cache_kernels(m) != CS_OK) {
     cudaFree(m->ws);
     cudaFree(m->wmem);
@@ -578,7 +601,7 @@ extern "C" cs_status cs_dit_forward(cs_model* m, const float* x, const int32_t* 
 static cs_status step_impl(cs_model* m, float* x, float* x_ref, float* delta, float* accum, uint8_t* has_ref, int N,
                            int k, int T, float t_cur, float t_next, float tau, int K_w, int K_c,
                            const uint8_t* force, uint8_t* skip, const float* target, float* scores, int* n_out,
-                           cudaStream_t s) {
+                           const void* tag_x, cudaStream_t s) {
   CS_REQUIRE(m && x && x_ref && delta && accum && has_ref && skip, "cs_search_step: null pointer");
   CS_REQUIRE(N > 0 && N <= m->cfg.max_batch, "cs_search_step: N=%d outside 1..max_batch=%d", N, m->cfg.max_batch);
   CS_REQUIRE(!target || scores, "cs_search_step: scoring needs scores");
@@ -588,48 +611,83 @@ static cs_status step_impl(cs_model* m, float* x, float* x_ref, float* delta, fl
   cudaEvent_t ev[2];
   const bool wf = k <= K_w || k > T - K_c;
   const bool tokens = m->tokens_update;
+  // the drift sums the previous step left apply when that step ran on the same state
+  // buffers and N and was step k - 1 (and each candidate's has_ref = 3 says they still
+  // belong to its latent)
+  auto& tag = m->carry_tag;
+  const bool carry_ok = tokens && tag.valid && tag.x == tag_x && tag.x_ref == x_ref && tag.delta == delta &&
+                        tag.accum == accum && tag.has_ref == has_ref && tag.N == N && tag.k + 1 == k;
+  tag.valid = false;
+  bool carried = false;   // decisions taken from carried drifts on a free step
   int n_c = N;
   const int32_t* idx = m->idx;
-  if (tokens && wf && !force) {
-    // warm-up / cool-down: every candidate computes and no drift is evaluated (Sec. 3.1);
-    // the computed update below writes the state (a = 0, has_ref = 1, skip = 0)
-    idx = m->idx_all;
-  } else {
-    // decisions + the update of skipped candidates; computed ones after the DiT
-    CS_TRY(record_begin(m, 3, s, ev));
-    CS_TRY(cs::decide_skip_run(x, x_ref, delta, accum, has_ref, N, D, k, T, t_cur, t_next, tau, K_w, K_c, force, skip,
-                               m->idx, m->n_compute, target, m->cache_ws,
-                               cs::StepScratch{m->cache_counter, m->cache_sidx}, m->err, s));
-    CS_TRY(record_end(m, 3, s, ev, 0.0));
+  auto read_decisions = [&]() -> cs_status {
     CS_CUDA(cudaMemcpyAsync(m->n_host, m->n_compute, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
     CS_CUDA(cudaMemcpyAsync(m->n_host + 1, m->err, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
     CS_CUDA(cudaStreamSynchronize(s));
-    n_c = m->n_host[0];
     if (m->n_host[1] != 0) {
       cs::set_error("cs_search_step: device error %d recorded before step %d", m->n_host[1], k);
       const int code = m->n_host[1];
       cudaMemsetAsync(m->err, 0, sizeof(int), s);
       return (cs_status)code;
     }
+    return CS_OK;
+  };
+  if (tokens && wf && !force) {
+    // warm-up / cool-down: every candidate computes and no drift is evaluated (Sec. 3.1);
+    // the computed update below writes the state (a = 0, has_ref = 3, skip = 0)
+    idx = m->idx_all;
+  } else if (tokens) {
+    // decisions + the update of skipped candidates; computed ones after the DiT
+    CS_TRY(record_begin(m, 3, s, ev));
+    CS_TRY(cs::carry_decide_skip_run(x, x_ref, delta, accum, has_ref, N, k, T, t_cur, t_next, tau, K_w, K_c, force,
+                                     skip, m->idx, m->n_compute, target, carry_ok, m->carry, m->err, s));
+    CS_TRY(record_end(m, 3, s, ev, 0.0));
+    CS_TRY(read_decisions());
+    carried = carry_ok && !wf;
+    if (m->n_host[0] < 0) {
+      // a cached candidate carries no drift (its state was written outside these calls):
+      // nothing was changed; take the drift pass
+      carried = false;
+      CS_TRY(record_begin(m, 3, s, ev));
+      CS_TRY(cs::carry_decide_skip_run(x, x_ref, delta, accum, has_ref, N, k, T, t_cur, t_next, tau, K_w, K_c, force,
+                                       skip, m->idx, m->n_compute, target, false, m->carry, m->err, s));
+      CS_TRY(record_end(m, 3, s, ev, 0.0));
+      CS_TRY(read_decisions());
+    }
+    n_c = m->n_host[0];
+  } else {
+    CS_TRY(record_begin(m, 3, s, ev));
+    CS_TRY(cs::decide_skip_run(x, x_ref, delta, accum, has_ref, N, D, k, T, t_cur, t_next, tau, K_w, K_c, force, skip,
+                               m->idx, m->n_compute, target, m->cache_ws,
+                               cs::StepScratch{m->cache_counter, m->cache_sidx}, m->err, s));
+    CS_TRY(record_end(m, 3, s, ev, 0.0));
+    CS_TRY(read_decisions());
+    n_c = m->n_host[0];
   }
   if (n_out) *n_out = n_c;
   CS_TRY(dit_forward_impl(m, x, idx, n_c, N, 1, t_cur, tokens ? nullptr : m->v, s));
   // algorithmic bytes of indicator + update (each tensor read or written once):
   //   skipped: read x, x_ref, Delta, write x                                 16 D
-  //   computed: read x, v (+ x_ref on a free step), write x, Delta, x_ref    20 D (24 D)
+  //   computed: read x, v, write x, Delta, x_ref                             20 D
+  //   (+ read x_ref for the drift of a free step whose drift was not carried: 24 D)
   const double skipped = N - n_c;
-  double bytes = skipped * 16.0 * D + n_c * (wf ? 20.0 : 24.0) * D;
+  double bytes = skipped * 16.0 * D + n_c * ((wf || carried) ? 20.0 : 24.0) * D;
   if (target) bytes += 4.0 * D * N;
-  if (n_c == 0 && !target) return add_work(m, 3, bytes);   // the decision pass did the whole update
+  if (n_c == 0 && !target) {
+    // the decision pass did the whole update
+    if (tokens) tag = {tag_x, x_ref, delta, accum, has_ref, N, k, true};
+    return add_work(m, 3, bytes);
+  }
   CS_TRY(record_begin(m, 3, s, ev));
-  float* spart = static_cast<float*>(m->cache_ws) + (size_t)N * ((D + 8191) / 8192) * 2;
   if (tokens) {
-    CS_TRY(cs::apply_tokens_run(x, x_ref, delta, accum, has_ref, skip, m->hout, idx, n_c, N, c.C, c.F, c.H, c.W,
-                                t_cur, t_next, target, scores, spart, m->tpart, N, m->err, s));
-  } else if (n_c > 0 || target) {
+    CS_TRY(cs::carry_apply_tokens_run(x, x_ref, delta, accum, has_ref, skip, m->hout, idx, n_c, N, c.C, c.F, c.H, c.W,
+                                      k, t_cur, t_next, target, scores, m->carry, N, m->err, s));
+  } else {
     CS_TRY(cs_cache_apply_computed(x, x_ref, delta, m->v, skip, N, D, t_cur, t_next, target, scores, m->cache_ws, s));
   }
   CS_TRY(record_end(m, 3, s, ev, bytes));
+  if (tokens) tag = {tag_x, x_ref, delta, accum, has_ref, N, k, true};
   return CS_OK;
 }
 
@@ -638,7 +696,7 @@ extern "C" cs_status cs_search_step(cs_model* m, float* x, float* x_ref, float* 
                                     int K_w, int K_c, const uint8_t* force, uint8_t* skip, const float* target,
                                     float* scores, int* n_computed, cudaStream_t s) {
   return step_impl(m, x, x_ref, delta, accum, has_ref, N, k, T, t_cur, t_next, tau, K_w, K_c, force, skip, target,
-                   scores, n_computed, s);
+                   scores, n_computed, x, s);
 }
 
 extern "C" cs_status cs_search_step_cfg(cs_model* m, float* x, float* x_ref, float* delta, float* accum,
@@ -650,6 +708,7 @@ extern "C" cs_status cs_search_step_cfg(cs_model* m, float* x, float* x_ref, flo
              m->cfg.max_batch);
   CS_REQUIRE(m->text_set && m->null_text_set, "cs_search_step_cfg: set both text contexts first");
   CS_REQUIRE(!target || scores, "cs_search_step_cfg: scoring needs scores");
+  m->carry_tag.valid = false;   // the guided step carries no drift
   const long long D = m->D;
   cudaEvent_t ev[2];
   const bool wf = k <= K_w || k > T - K_c;
@@ -687,7 +746,7 @@ extern "C" cs_status cs_search_step_host(cs_model* m, float* x_host, float* x_re
   const size_t bytes = (size_t)N * m->D * sizeof(float);
   CS_CUDA(cudaMemcpyAsync(m->x_host_stage, x_host, bytes, cudaMemcpyHostToDevice, s));
   CS_TRY(step_impl(m, m->x_host_stage, x_ref, delta, accum, has_ref, N, k, T, t_cur, t_next, tau, K_w, K_c, nullptr,
-                   m->skip_tmp, nullptr, nullptr, n_computed, s));
+                   m->skip_tmp, nullptr, nullptr, n_computed, x_host, s));
   CS_CUDA(cudaMemcpyAsync(x_host, m->x_host_stage, bytes, cudaMemcpyDeviceToHost, s));
   CS_CUDA(cudaMemcpyAsync(skip_host, m->skip_tmp, N, cudaMemcpyDeviceToHost, s));
   CS_CUDA(cudaStreamSynchronize(s));

@@ -23,6 +23,7 @@
 namespace cs {
 
 constexpr int kCacheThreads = 256;
+constexpr int kCacheWarps = kCacheThreads / 32;
 constexpr long long kChunkElems = 8192;    // elements of one candidate per CTA (multiple of 4*256)
 
 __host__ __device__ inline int cache_chunks(long long D) {
@@ -562,15 +563,17 @@ __global__ void __launch_bounds__(kCacheThreads) drift_decide_kernel(
 // to be still in L2).
 template <bool kScore>
 __global__ void __launch_bounds__(kCacheThreads, 4) skip_update_kernel(
-    float* __restrict__ x, const float* __restrict__ delta, const int32_t* __restrict__ sidx, int N, long long D,
+    float* __restrict__ x, const float* __restrict__ delta, const int32_t* sidx, int N, long long D,
     int nch, float h, float t_next, const float* __restrict__ target, float* __restrict__ spart) {
   __shared__ float red[1][32];
-  pdl_wait_primary();        // the decisions (and every write of the first kernel) are visible
-  const int items = sidx[N] * nch;
+  // the decisions (and every write of the first kernel) are visible after the wait; the
+  // list is read through L2 (a read-only cached load could be placed before the wait)
+  pdl_wait_primary();
+  const int items = __ldcg(sidx + N) * nch;
   const int per = (items + gridDim.x - 1) / gridDim.x;
   const int it1 = items - blockIdx.x * per, it0 = max(0, it1 - per);
   for (int item = it1 - 1; item >= it0; --item) {
-    const int i = sidx[item / nch], c = item % nch;
+    const int i = __ldcg(sidx + item / nch), c = item % nch;
     const long long lo = (long long)c * kChunkElems, hi = min(D, lo + kChunkElems);
     float* xi = x + (long long)i * D + lo;
     const float* di = delta + (long long)i * D + lo;
@@ -620,6 +623,328 @@ __global__ void __launch_bounds__(kCacheThreads, 4) skip_update_kernel(
       block_sum<1>(acc, red);
       if (threadIdx.x == 0) spart[(long long)i * nch + c] = acc[0];
       block_sync();
+    }
+  }
+}
+
+// ---------------------------------------------------------- carried drift ----
+// The drift of Eq. indicator at step k needs ||x - x_ref|| and ||x_ref|| of the latent a
+// candidate holds at step k.  That latent is written by the update of step k - 1, which
+// has x_next and the x_ref it leaves in registers at that moment, so the update kernels
+// also leave the two squared norms, per candidate, for the next step: the drift is
+// carried.  A step whose cached candidates all carry one takes its decisions without
+// reading x or x_ref, and its skip update is the one pass over a skipped candidate's
+// state: read x, Delta and x_ref, write x, and leave the sums for step k + 1.
+// has_ref = 3 (bit 1 set) marks a candidate whose carried sums belong to its current x
+// and x_ref; every other writer of the state leaves has_ref = 1.
+//
+// The partial pairs of a candidate are summed by whichever CTA completes its last chunk
+// or token row (per-candidate completion counter, left at zero), in a fixed order that
+// does not depend on that CTA, so the carried value depends on the candidate alone.
+struct CarryOut {
+  float2* part;        // [cap][P] partial pairs of the candidate's chunk warps or token rows
+  int P;
+  unsigned* cnt;       // [cap] completion counts (zero between calls)
+  float2* drift_out;   // [cap] (sum (x_next - x_ref)^2, sum x_ref^2) for the next step
+};
+
+__device__ __forceinline__ void carry_finalize(const CarryOut& c, int i, int n, float (*red)[32]) {
+  __threadfence();
+  float v[2] = {0.f, 0.f};
+  const float2* p = c.part + (long long)i * c.P;
+  for (int q = threadIdx.x; q < n; q += kCacheThreads) {
+    const float2 a = __ldcg(p + q);
+    v[0] += a.x;
+    v[1] += a.y;
+  }
+  block_sum<2>(v, red);
+  if (threadIdx.x == 0) {
+    c.drift_out[i] = make_float2(v[0], v[1]);
+    c.cnt[i] = 0u;
+  }
+  block_sync();
+}
+
+// Decision flags of the carried form (per candidate, in shared memory).
+constexpr uint8_t kFlCompute = 1, kFlNonFinite = 2, kFlArg = 4, kFlBad = 8;
+
+// The decision of candidate i from the drift carried into this step (Sec. 3.1): free step
+// with a cached reference: a += drift, compute iff tau <= 0 or a > tau; inside the window
+// or with an empty cache: compute, no drift; then the forced mask.  kFlBad: a cached
+// candidate without a carried drift on a free step.  Every caller gets the same bits.
+__device__ __forceinline__ uint8_t decide_carried(int i, int wf, float tau, const uint8_t* __restrict__ has_ref,
+                                                  const float* __restrict__ accum, const float2* __restrict__ drift_in,
+                                                  const uint8_t* __restrict__ force, float& a) {
+  const uint8_t hr = has_ref[i];
+  const bool had = hr != 0;
+  bool compute = true;
+  uint8_t fl = 0;
+  a = accum[i];
+  if (!wf && had) {
+    if (!(hr & 2)) {
+      fl |= kFlBad;
+    } else {
+      const float2 s2 = drift_in[i];
+      const float drift = drift_of(s2.x, s2.y);
+      if (!isfinite(drift)) {
+        fl |= kFlNonFinite;
+      } else {
+        a = a + drift;
+        compute = (tau <= 0.f) || (a > tau);
+      }
+    }
+  }
+  if (force) {
+    const bool f = force[i] != 0;
+    if (!f && !had) fl |= kFlArg;
+    else compute = f;
+  }
+  if (compute) a = 0.f;
+  return fl | (compute ? kFlCompute : 0);
+}
+
+// TMA ring of the skip update: a unit is 4096 elements of one candidate; one stage holds a
+// unit of x, Delta and x_ref (48 KB); four stages keep 192 KB per SM in flight whatever
+// the registers of the consuming threads.
+constexpr int kUnitElems = 4096;
+constexpr int kSkipStages = 4;
+constexpr int kSkipStageFloats = 3 * kUnitElems;
+constexpr size_t kSkipRingBytes = (size_t)kSkipStages * kSkipStageFloats * sizeof(float);
+
+__host__ __device__ inline int carry_units(long long D) {
+  long long u = (D + kUnitElems - 1) / kUnitElems;
+  return (int)(u < 1 ? 1 : u);
+}
+
+__host__ inline size_t carry_skip_smem(int N) {
+  return kSkipRingBytes + (size_t)(3 * N + 15) / 16 * 16;   // + skipped list (16-bit) and flags
+}
+
+// The skip update of cs_search_step with the carried drift, one CTA per SM.  Per skipped
+// candidate and unit: x_next = x + h (x + Delta) (Eq. skip + Eq. euler), written back, and
+// the unit's partial pair of the next step's drift, (x_next - x_ref)^2 and x_ref^2 (thread
+// sums, warp trees, then the eight warps in order); with a target, the unit's score
+// partial.  Thread 0 keeps the ring full (cp.async.bulk, one mbarrier per stage, waits
+// bounded); the units of the CTA's contiguous share of (skipped candidate, unit) items are
+// consumed in order.  When the CTA finishes its units of a candidate it counts them in;
+// the CTA that completes the candidate sums its unit pairs (warp 0, fixed order) into
+// carry.drift_out.
+//  kDecide  every CTA takes the same decisions from the same inputs (decide_carried) and
+//           so knows the skipped list; every CTA counts itself in on one arrival counter,
+//           and the CTA that arrives last (after every CTA has read the state) writes
+//           accum, has_ref (3 for skipped candidates, whose new sums are complete), the
+//           skip mask and the list of computing candidates, and leaves the counter at
+//           zero.  A free step on which a cached candidate carries no drift changes
+//           nothing and reports *n_compute = -1: the caller then runs the drift pass.
+//  !kDecide the decisions and the skipped list come from drift_decide_kernel (launched
+//           before this one with programmatic stream serialisation); the CTA completing a
+//           candidate sets its has_ref to 3.
+template <bool kScore, bool kDecide>
+__global__ void __launch_bounds__(kCacheThreads, 1) carry_skip_kernel(
+    float* __restrict__ x, const float* __restrict__ xr, const float* __restrict__ delta, float* __restrict__ accum,
+    uint8_t* __restrict__ has_ref, int N, long long D, int nun, int wf, float tau, const uint8_t* __restrict__ force,
+    uint8_t* __restrict__ skip_mask, int32_t* __restrict__ idx, int32_t* __restrict__ n_compute,
+    const int32_t* sidx_in, const float2* __restrict__ drift_in, CarryOut carry,
+    unsigned* __restrict__ counter, float h, float t_next, const float* __restrict__ target,
+    float* __restrict__ spart, int* err) {
+  constexpr int NV = kScore ? 3 : 2;
+  extern __shared__ __align__(128) uint8_t smem[];
+  float* ring = reinterpret_cast<float*>(smem);
+  uint16_t* s_list = reinterpret_cast<uint16_t*>(smem + kSkipRingBytes);
+  uint8_t* s_flag = reinterpret_cast<uint8_t*>(s_list + N);
+  __shared__ uint64_t full[kSkipStages];
+  __shared__ float red[2][NV][kCacheWarps];
+  __shared__ int s_ns, s_bad, s_last, s_abort;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) {
+    for (int q = 0; q < kSkipStages; ++q) mbar_init(&full[q], 1);
+    fence_mbar_init();
+    s_bad = 0;
+    s_abort = 0;
+  }
+  block_sync();
+  int ns;
+  if (kDecide) {
+    for (int i = threadIdx.x; i < N; i += kCacheThreads) {
+      float a;
+      const uint8_t fl = decide_carried(i, wf, tau, has_ref, accum, drift_in, force, a);
+      s_flag[i] = fl;
+      if (fl & kFlBad) s_bad = 1;
+    }
+    block_sync();
+    if (warp == 0) {
+      int n = 0;
+      for (int base = 0; base < N; base += 32) {
+        const int k = base + lane;
+        const bool sk = k < N && !(s_flag[k] & kFlCompute);
+        const unsigned b = __ballot_sync(0xffffffffu, sk);
+        if (sk) s_list[n + __popc(b & ((1u << lane) - 1u))] = (uint16_t)k;
+        n += __popc(b);
+      }
+      if (lane == 0) s_ns = s_bad ? 0 : n;
+    }
+    block_sync();
+    ns = s_ns;
+  } else {
+    // the decisions (and every write of the drift pass) are visible after the wait; read
+    // them through L2 (a read-only cached load could be placed before the wait)
+    pdl_wait_primary();
+    ns = __ldcg(sidx_in + N);
+    for (int q = threadIdx.x; q < ns; q += kCacheThreads) s_list[q] = (uint16_t)__ldcg(sidx_in + q);
+    block_sync();
+  }
+  // this CTA's items: a balanced contiguous share of the (skipped candidate, unit) items
+  const long long items = (long long)ns * nun;
+  const int it0 = (int)(items * blockIdx.x / gridDim.x), it1 = (int)(items * (blockIdx.x + 1) / gridDim.x);
+  const int n_it = it1 - it0;
+  auto issue = [&](int k) {                       // thread 0: item k of this CTA into stage k % S
+    const int it = it0 + k, sq = it / nun, u = it - sq * nun, i = s_list[sq];
+    const long long lo = (long long)u * kUnitElems;
+    const uint32_t bytes = (uint32_t)(min((long long)kUnitElems, D - lo) * sizeof(float));
+    float* st = ring + (size_t)(k % kSkipStages) * kSkipStageFloats;
+    uint64_t* bar = &full[k % kSkipStages];
+    mbar_arrive_expect_tx(bar, 3 * bytes);
+    bulk_load_1d(st, x + (long long)i * D + lo, bytes, bar);
+    bulk_load_1d(st + kUnitElems, delta + (long long)i * D + lo, bytes, bar);
+    bulk_load_1d(st + 2 * kUnitElems, xr + (long long)i * D + lo, bytes, bar);
+  };
+  if (threadIdx.x == 0)
+    for (int k = 0; k < kSkipStages && k < n_it; ++k) issue(k);
+  int done_from = 0;                              // first item of the current candidate's run
+  int n_consumed = n_it;
+  for (int k = 0; k < n_it; ++k) {
+    const int sq = (it0 + k) / nun, u = it0 + k - sq * nun, i = s_list[sq];
+    if (!mbar_wait(&full[k % kSkipStages], (uint32_t)(k / kSkipStages) & 1u, (volatile int*)&s_abort, err)) {
+      n_consumed = k;
+      break;
+    }
+    const float* st = ring + (size_t)(k % kSkipStages) * kSkipStageFloats;
+    const float4* sx = reinterpret_cast<const float4*>(st);
+    const float4* sd = reinterpret_cast<const float4*>(st + kUnitElems);
+    const float4* sr = reinterpret_cast<const float4*>(st + 2 * kUnitElems);
+    const long long lo = (long long)u * kUnitElems;
+    const int n4 = (int)(min((long long)kUnitElems, D - lo) >> 2);
+    float4* xo = reinterpret_cast<float4*>(x + (long long)i * D + lo);
+    const float4* y4 = kScore ? reinterpret_cast<const float4*>(target + lo) : nullptr;
+    float acc[NV];
+#pragma unroll
+    for (int q = 0; q < NV; ++q) acc[q] = 0.f;
+#pragma unroll 4
+    for (int q = threadIdx.x; q < n4; q += kCacheThreads) {
+      const float4 xv = sx[q], dv = sd[q], rv = sr[q];
+      const float4 vu = make_float4(xv.x + dv.x, xv.y + dv.y, xv.z + dv.z, xv.w + dv.w);            // Eq. skip
+      const float4 xn = make_float4(xv.x + h * vu.x, xv.y + h * vu.y, xv.z + h * vu.z, xv.w + h * vu.w);  // Eq. euler
+      __stcs(xo + q, xn);
+      const float d0 = xn.x - rv.x, d1 = xn.y - rv.y, d2 = xn.z - rv.z, d3 = xn.w - rv.w;
+      acc[0] += d0 * d0 + d1 * d1 + d2 * d2 + d3 * d3;
+      acc[1] += rv.x * rv.x + rv.y * rv.y + rv.z * rv.z + rv.w * rv.w;
+      if (kScore) {
+        const float4 y = __ldg(y4 + q);
+        const float e0 = xn.x - t_next * vu.x - y.x, e1 = xn.y - t_next * vu.y - y.y;
+        const float e2 = xn.z - t_next * vu.z - y.z, e3 = xn.w - t_next * vu.w - y.w;
+        acc[2] += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < NV; ++q) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) acc[q] += __shfl_xor_sync(0xffffffffu, acc[q], o);
+    }
+    if (lane == 0) {
+#pragma unroll
+      for (int q = 0; q < NV; ++q) red[k & 1][q][warp] = acc[q];
+    }
+    block_sync();                                 // every thread is done with stage k % S
+    if (warp == 0) {
+      int fin = 0;
+      if (lane == 0) {
+        float p[NV];
+#pragma unroll
+        for (int q = 0; q < NV; ++q) {
+          p[q] = 0.f;
+#pragma unroll
+          for (int w = 0; w < kCacheWarps; ++w) p[q] += red[k & 1][q][w];
+        }
+        carry.part[(long long)i * carry.P + u] = make_float2(p[0], p[1]);
+        if (kScore) spart[(long long)i * nun + u] = p[NV - 1];
+        if (k + kSkipStages < n_it) issue(k + kSkipStages);
+        const bool last_of_run = k + 1 == n_it || (it0 + k + 1) / nun != sq;
+        if (last_of_run) {
+          const unsigned run = (unsigned)(k - done_from + 1);
+          __threadfence();
+          fin = atomicAdd(carry.cnt + i, run) + run == (unsigned)nun;
+        }
+      }
+      fin = __shfl_sync(0xffffffffu, fin, 0);
+      if (fin) {   // the candidate is complete: warp 0 sums its unit pairs in a fixed order
+        __threadfence();
+        const float2* pp = carry.part + (long long)i * carry.P;
+        float s0 = 0.f, s1 = 0.f;
+        for (int q = lane; q < nun; q += 32) {
+          const float2 a = __ldcg(pp + q);
+          s0 += a.x;
+          s1 += a.y;
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          s0 += __shfl_xor_sync(0xffffffffu, s0, o);
+          s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+        }
+        if (lane == 0) {
+          carry.drift_out[i] = make_float2(s0, s1);
+          carry.cnt[i] = 0u;
+          if (!kDecide) has_ref[i] = 3;
+        }
+      }
+    }
+    if (k + 1 < n_it && (it0 + k + 1) / nun != sq) done_from = k + 1;
+  }
+  if (s_abort && threadIdx.x == 0) {
+    // a wait ran out: let the copies already issued (items n_consumed .. n_consumed + S - 1
+    // at most) land before the CTA's memory goes
+    for (int k = n_consumed; k < n_it && k < n_consumed + kSkipStages; ++k)
+      mbar_wait_teardown(&full[k % kSkipStages], (uint32_t)(k / kSkipStages) & 1u);
+  }
+  if (!kDecide) return;
+  // arrival: the CTA that arrives last (every CTA has read the state by then) writes it
+  if (threadIdx.x == 0) {
+    __threadfence();
+    s_last = atomicAdd(counter, 1u) == gridDim.x - 1;
+  }
+  block_sync();
+  if (!s_last) return;
+  __threadfence();
+  if (s_bad) {
+    if (threadIdx.x == 0) {
+      *n_compute = -1;
+      *counter = 0u;
+    }
+    return;
+  }
+  for (int i = threadIdx.x; i < N; i += kCacheThreads) {
+    float a;
+    const uint8_t fl = decide_carried(i, wf, tau, has_ref, accum, drift_in, force, a);
+    const bool compute = fl & kFlCompute;
+    if (fl & kFlNonFinite) record_error(err, CS_ERR_NONFINITE);
+    if (fl & kFlArg) record_error(err, CS_ERR_ARG);
+    s_flag[i] = fl;
+    accum[i] = a;
+    skip_mask[i] = compute ? 0 : 1;
+    has_ref[i] = compute ? 1 : 3;
+  }
+  block_sync();
+  if (warp == 0) {
+    int nc = 0;
+    for (int base = 0; base < N; base += 32) {
+      const int k = base + lane;
+      const bool comp = k < N && (s_flag[k] & kFlCompute);
+      const unsigned b = __ballot_sync(0xffffffffu, comp);
+      if (comp) idx[nc + __popc(b & ((1u << lane) - 1u))] = k;
+      nc += __popc(b);
+    }
+    if (lane == 0) {
+      *n_compute = nc;
+      *counter = 0u;
     }
   }
 }
@@ -685,16 +1010,24 @@ __global__ void __launch_bounds__(kCacheThreads) apply_computed_kernel(
 //   Delta = v - x,  x_ref = x,  x += (t_next - t_cur) v,  accum = 0, has_ref = 1, skip = 0.
 // One CTA per (token row (f, h/2), computed candidate): the row's W/2 tokens x P features
 // (contiguous in hout) are staged in shared memory as one float4 per (w/4, c, h&1) that
-// holds v at w..w+3, so hout and the four state tensors all move in 16-byte accesses.
+// holds v at w..w+3, so hout and the four state tensors all move in 16-byte accesses; a
+// thread issues all its loads of a phase before it uses the first.
 // The score partial of a tile is a fixed-order block sum (independent of the batch).
-template <bool kScore>
+// With kCarry the CTA also leaves the row's pair of the next step's drift terms
+// (x_next - x_ref_new = x_next - x, and x_ref_new = x, both in registers here) for
+// carry_rows_finalize_kernel, and has_ref = 3.
+constexpr int kVelUnroll = 4;   // float4 loads in flight per thread and phase (rows up to 1024 of them)
+
+template <bool kScore, bool kCarry>
 __global__ void __launch_bounds__(kCacheThreads) velocity_update_kernel(
     const float* __restrict__ hout, const int32_t* __restrict__ idx, int C, int F, int H, int W,
     float* __restrict__ x, float* __restrict__ xr, float* __restrict__ delta, float* __restrict__ accum,
     uint8_t* __restrict__ has_ref, uint8_t* __restrict__ skip_mask, float h, float t_next,
-    const float* __restrict__ target, float* __restrict__ tpart, long long idx_limit, int* err) {
+    const float* __restrict__ target, float* __restrict__ tpart, CarryOut carry, long long idx_limit, int* err) {
+  constexpr int NV = kCarry ? 3 : 1;              // score, then the carried pair
   extern __shared__ float4 s_v[];                 // [W/4][2C + 1]: the +1 staggers the banks
-  __shared__ float red[1][32];
+  __shared__ float red[3][32];
+  if (kCarry) pdl_launch_dependents();            // the finalize may be scheduled while this drains
   const int H2 = H / 2, W2 = W / 2, W4 = W / 4, S = 2 * C + 1;
   const int row = blockIdx.x, j = blockIdx.y;     // row = f * H/2 + h/2
   const int f = row / H2, hh = row % H2;
@@ -703,23 +1036,41 @@ __global__ void __launch_bounds__(kCacheThreads) velocity_update_kernel(
   const long long D = (long long)C * F * H * W;
   const long long L = (long long)F * H2 * W2;
   const float4* src = reinterpret_cast<const float4*>(hout + ((long long)j * L + (long long)row * W2) * (4 * C));
-  for (int q = threadIdx.x; q < W2 * C; q += kCacheThreads) {
-    const float4 a = __ldcs(src + q);             // features 4c..4c+3 of token T: (ph, pw) = 00 01 10 11
+  auto stage = [&](int q, float4 a) {             // features 4c..4c+3 of token T: (ph, pw) = 00 01 10 11
     const int T = q / C, c = q % C;
     float2* d = reinterpret_cast<float2*>(&s_v[(T >> 1) * S + 2 * c]) + (T & 1);
     d[0] = make_float2(a.x, a.y);                 // h even: w = 2T, 2T + 1
     d[2] = make_float2(a.z, a.w);                 // h odd
+  };
+  const int nq = W2 * C;
+  {
+    float4 a[kVelUnroll];
+#pragma unroll
+    for (int u = 0; u < kVelUnroll; ++u) {
+      const int q = threadIdx.x + u * kCacheThreads;
+      if (q < nq) a[u] = __ldcs(src + q);
+    }
+#pragma unroll
+    for (int u = 0; u < kVelUnroll; ++u) {
+      const int q = threadIdx.x + u * kCacheThreads;
+      if (q < nq) stage(q, a[u]);
+    }
+    for (int q = threadIdx.x + kVelUnroll * kCacheThreads; q < nq; q += kCacheThreads) stage(q, __ldcs(src + q));
   }
   block_sync();
   float* xi = x + (long long)i * D;
   float* ri = xr + (long long)i * D;
   float* di = delta + (long long)i * D;
-  float acc[1] = {0.f};
-  for (int q = threadIdx.x; q < 2 * C * W4; q += kCacheThreads) {
-    const int w4 = q % W4, cp = q / W4;           // cp = 2c + (h & 1)
-    const long long e = (((long long)(cp >> 1) * F + f) * H + 2 * hh + (cp & 1)) * W + 4 * w4;
+  float acc[NV];
+#pragma unroll
+  for (int q = 0; q < NV; ++q) acc[q] = 0.f;
+  auto offset = [&](int q, int& cp, int& w4) {
+    w4 = q % W4;
+    cp = q / W4;                                  // cp = 2c + (h & 1)
+    return (((long long)(cp >> 1) * F + f) * H + 2 * hh + (cp & 1)) * W + 4 * w4;
+  };
+  auto update = [&](long long e, int cp, int w4, float4 xv) {
     const float4 vu = s_v[w4 * S + cp];
-    const float4 xv = __ldcs(reinterpret_cast<const float4*>(xi + e));
     __stcs(reinterpret_cast<float4*>(di + e), make_float4(vu.x - xv.x, vu.y - xv.y, vu.z - xv.z, vu.w - xv.w));
     __stcs(reinterpret_cast<float4*>(ri + e), xv);
     const float4 xn = make_float4(xv.x + h * vu.x, xv.y + h * vu.y, xv.z + h * vu.z, xv.w + h * vu.w);
@@ -730,16 +1081,60 @@ __global__ void __launch_bounds__(kCacheThreads) velocity_update_kernel(
       const float e2 = xn.z - t_next * vu.z - y.z, e3 = xn.w - t_next * vu.w - y.w;
       acc[0] += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
     }
+    if (kCarry) {   // the next step's drift terms: x_next - x_ref_new (as stored), x_ref_new
+      const float d0 = xn.x - xv.x, d1 = xn.y - xv.y, d2 = xn.z - xv.z, d3 = xn.w - xv.w;
+      acc[NV - 2] += d0 * d0 + d1 * d1 + d2 * d2 + d3 * d3;
+      acc[NV - 1] += xv.x * xv.x + xv.y * xv.y + xv.z * xv.z + xv.w * xv.w;
+    }
+  };
+  const int nu = 2 * C * W4;
+  {
+    float4 xv[kVelUnroll];
+    long long e[kVelUnroll];
+    int cp[kVelUnroll], w4[kVelUnroll];
+#pragma unroll
+    for (int u = 0; u < kVelUnroll; ++u) {
+      const int q = threadIdx.x + u * kCacheThreads;
+      if (q < nu) {
+        e[u] = offset(q, cp[u], w4[u]);
+        xv[u] = __ldcs(reinterpret_cast<const float4*>(xi + e[u]));
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kVelUnroll; ++u)
+      if (threadIdx.x + u * kCacheThreads < nu) update(e[u], cp[u], w4[u], xv[u]);
+    for (int q = threadIdx.x + kVelUnroll * kCacheThreads; q < nu; q += kCacheThreads) {
+      int c2, w2;
+      const long long e2 = offset(q, c2, w2);
+      update(e2, c2, w2, __ldcs(reinterpret_cast<const float4*>(xi + e2)));
+    }
   }
-  if (kScore) {
-    block_sum<1>(acc, red);
-    if (threadIdx.x == 0) tpart[(long long)i * gridDim.x + row] = acc[0];
+  if (kScore || kCarry) {
+    block_sum<NV>(acc, red);
+    if (threadIdx.x == 0) {
+      if (kScore) tpart[(long long)i * gridDim.x + row] = acc[0];
+      if (kCarry) carry.part[(long long)i * carry.P + row] = make_float2(acc[NV - 2], acc[NV - 1]);
+    }
   }
   if (row == 0 && threadIdx.x == 0) {
     accum[i] = 0.f;
-    has_ref[i] = 1;
+    has_ref[i] = kCarry ? 3 : 1;
     skip_mask[i] = 0;
   }
+}
+
+// The computed candidates' carried drift: one CTA per computed candidate sums its token
+// rows' pairs (carry_finalize, fixed order).  Launched after velocity_update_kernel with
+// programmatic stream serialisation: scheduled while the update drains, it waits for its
+// completion before reading.
+__global__ void __launch_bounds__(kCacheThreads) carry_rows_finalize_kernel(const int32_t* __restrict__ idx,
+                                                                           int ntiles, CarryOut carry,
+                                                                           long long idx_limit, int* err) {
+  __shared__ float red[2][32];
+  pdl_wait_primary();
+  const int i = idx[blockIdx.x];
+  if (!index_ok(i, idx_limit, err)) return;      // uniform over the CTA
+  carry_finalize(carry, i, ntiles, red);
 }
 
 // Scores when the two kinds of candidates left their partials in different groupings:
@@ -799,7 +1194,7 @@ __global__ void __launch_bounds__(kCacheThreads) beam_refill_kernel(
   }
   if (c == 0 && threadIdx.x == 0) {
     da[slot] = sa[src];
-    dh[slot] = sh[src];
+    dh[slot] = sh[src] ? 1 : 0;   // a carried drift belongs to the source slot's latent: not copied
   }
 }
 
@@ -998,8 +1393,12 @@ cs_status decide_skip_run(float* x, const float* x_ref, const float* delta, floa
 cs_status load_cache_kernels() {
   const void* fns[] = {
       (const void*)drift_decide_kernel,          (const void*)skip_update_kernel<true>,
-      (const void*)skip_update_kernel<false>,    (const void*)velocity_update_kernel<true>,
-      (const void*)velocity_update_kernel<false>, (const void*)score_finalize_split_kernel,
+      (const void*)skip_update_kernel<false>,    (const void*)velocity_update_kernel<true, false>,
+      (const void*)velocity_update_kernel<false, false>, (const void*)score_finalize_split_kernel,
+      (const void*)velocity_update_kernel<true, true>, (const void*)velocity_update_kernel<false, true>,
+      (const void*)carry_skip_kernel<true, true>,  (const void*)carry_skip_kernel<false, true>,
+      (const void*)carry_skip_kernel<true, false>, (const void*)carry_skip_kernel<false, false>,
+      (const void*)carry_rows_finalize_kernel,
       (const void*)decide_finalize_kernel,       (const void*)decide_all_compute_kernel,
       (const void*)drift_partials_kernel,        (const void*)apply_computed_kernel<true>,
       (const void*)apply_computed_kernel<false>, (const void*)score_finalize_kernel,
@@ -1023,18 +1422,199 @@ cs_status apply_tokens_run(float* x, float* x_ref, float* delta, float* accum, u
   if (n_c > 0) {
     const dim3 grid(ntiles, n_c);
     if (target)
-      velocity_update_kernel<true><<<grid, kCacheThreads, smem, stream>>>(hout, idx, C, F, H, W, x, x_ref, delta,
-                                                                         accum, has_ref, skip_mask, h, t_next, target,
-                                                                         tpart, idx_limit, err);
+      velocity_update_kernel<true, false><<<grid, kCacheThreads, smem, stream>>>(
+          hout, idx, C, F, H, W, x, x_ref, delta, accum, has_ref, skip_mask, h, t_next, target, tpart, CarryOut{},
+          idx_limit, err);
     else
-      velocity_update_kernel<false><<<grid, kCacheThreads, smem, stream>>>(hout, idx, C, F, H, W, x, x_ref, delta,
-                                                                          accum, has_ref, skip_mask, h, t_next,
-                                                                          nullptr, nullptr, idx_limit, err);
+      velocity_update_kernel<false, false><<<grid, kCacheThreads, smem, stream>>>(
+          hout, idx, C, F, H, W, x, x_ref, delta, accum, has_ref, skip_mask, h, t_next, nullptr, nullptr,
+          CarryOut{}, idx_limit, err);
     CS_LAUNCHED();
   }
   if (target) {
     score_finalize_split_kernel<<<(N + 3) / 4, 128, 0, stream>>>(spart, cache_chunks(D), tpart, ntiles, skip_mask, N,
                                                                  scores);
+    CS_LAUNCHED();
+  }
+  return CS_OK;
+}
+
+// ------------------------------------------------------------ carried form ----
+// Step workspace of the carried form for `cap` candidate slots, each part at a 256-byte
+// boundary: arrival counter; skipped list [cap + 1]; completion counts [cap]; carried
+// sums [2][cap] (float2, by the parity of the step that reads them); partial pairs
+// [cap][max(units, F*H/2)] (float2; units of 4096 elements); drift-pass partials
+// [cap][nch][2]; skipped candidates' score partials [cap][units]; computed candidates'
+// score partials [cap][F*H/2].
+struct StepLayout {
+  size_t counter, sidx, cnt, drift, part, dpart, spart, tpart, total;
+  int nch, nun, P;
+};
+
+static StepLayout step_layout(int cap, long long D, int ntiles) {
+  StepLayout L;
+  size_t o = 0;
+  auto take = [&o](size_t bytes) {
+    o = (o + 255) / 256 * 256;
+    const size_t at = o;
+    o += bytes;
+    return at;
+  };
+  L.nch = cache_chunks(D);
+  L.nun = carry_units(D);
+  L.P = L.nun > ntiles ? L.nun : ntiles;
+  L.counter = take(sizeof(unsigned));
+  L.sidx = take((size_t)(cap + 1) * sizeof(int32_t));
+  L.cnt = take((size_t)cap * sizeof(unsigned));
+  L.drift = take((size_t)2 * cap * sizeof(float2));
+  L.part = take((size_t)cap * L.P * sizeof(float2));
+  L.dpart = take((size_t)cap * L.nch * 2 * sizeof(float));
+  L.spart = take((size_t)cap * L.nun * sizeof(float));
+  L.tpart = take((size_t)cap * ntiles * sizeof(float));
+  L.total = (o + 255) / 256 * 256;
+  return L;
+}
+
+size_t carry_state_bytes(int cap, long long D, int ntiles) { return step_layout(cap, D, ntiles).total; }
+
+static CarryOut carry_out(const CarryState& cs, const StepLayout& L, int step_k) {
+  char* b = static_cast<char*>(cs.base);
+  return CarryOut{reinterpret_cast<float2*>(b + L.part), L.P, reinterpret_cast<unsigned*>(b + L.cnt),
+                  reinterpret_cast<float2*>(b + L.drift) + (size_t)((step_k + 1) & 1) * cs.cap};
+}
+
+// The skip kernels' shared memory (the ring plus the list of up to 4096 candidates) is
+// above the default limit: raised once per process for each instantiation.
+static cs_status carry_skip_attributes() {
+  static std::once_flag once;
+  static cudaError_t e = cudaSuccess;
+  std::call_once(once, [] {
+    const int bytes = (int)carry_skip_smem(4096);
+    const void* fns[] = {(const void*)carry_skip_kernel<true, true>, (const void*)carry_skip_kernel<false, true>,
+                         (const void*)carry_skip_kernel<true, false>, (const void*)carry_skip_kernel<false, false>};
+    for (const void* f : fns) {
+      const cudaError_t r = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+      if (r != cudaSuccess && e == cudaSuccess) e = r;
+    }
+  });
+  CS_CUDA(e);
+  return CS_OK;
+}
+
+cs_status carry_decide_skip_run(float* x, const float* x_ref, const float* delta, float* accum, uint8_t* has_ref,
+                                int N, int step_k, int T, float t_cur, float t_next, float tau, int K_w, int K_c,
+                                const uint8_t* force, uint8_t* skip_mask, int32_t* idx, int32_t* n_compute,
+                                const float* target, bool carried, const CarryState& cs, int* err,
+                                cudaStream_t stream) {
+  const long long D = cs.D;
+  const int wf = window_forced(step_k, T, K_w, K_c) ? 1 : 0;
+  if (wf && !force) {
+    decide_all_compute_kernel<<<1, 256, 0, stream>>>(accum, has_ref, N, skip_mask, idx, n_compute);
+    CS_LAUNCHED();
+    return CS_OK;
+  }
+  const StepLayout L = step_layout(cs.cap, D, cs.ntiles);
+  char* b = static_cast<char*>(cs.base);
+  unsigned* counter = reinterpret_cast<unsigned*>(b + L.counter);
+  int32_t* sidx = reinterpret_cast<int32_t*>(b + L.sidx);
+  const CarryOut co = carry_out(cs, L, step_k);
+  const float2* din = reinterpret_cast<const float2*>(b + L.drift) + (size_t)(step_k & 1) * cs.cap;
+  float* spart = reinterpret_cast<float*>(b + L.spart);
+  const int nch = L.nch, nun = L.nun;
+  const float h = t_next - t_cur;
+  const size_t smem = carry_skip_smem(N);
+  int grid = num_sms();                           // one CTA per SM (the ring takes its shared memory)
+  if (grid > N * nun) grid = N * nun;
+  CS_TRY(carry_skip_attributes());
+  if (carried || wf) {
+    // decisions from the carried drift (none is needed inside the window): one launch
+    if (target)
+      carry_skip_kernel<true, true><<<grid, kCacheThreads, smem, stream>>>(
+          x, x_ref, delta, accum, has_ref, N, D, nun, wf, tau, force, skip_mask, idx, n_compute, nullptr, din, co,
+          counter, h, t_next, target, spart, err);
+    else
+      carry_skip_kernel<false, true><<<grid, kCacheThreads, smem, stream>>>(
+          x, x_ref, delta, accum, has_ref, N, D, nun, wf, tau, force, skip_mask, idx, n_compute, nullptr, din, co,
+          counter, h, t_next, nullptr, nullptr, err);
+    CS_LAUNCHED();
+    return CS_OK;
+  }
+  // no carried drift: the drift pass decides, then the skip update follows it
+  const int items = N * nch;
+  int g1 = resident_grid((const void*)drift_decide_kernel, N);
+  if (g1 > items) g1 = items;
+  drift_decide_kernel<<<g1, kCacheThreads, N, stream>>>(x, x_ref, accum, has_ref, N, D, nch, tau, force, skip_mask,
+                                                       idx, n_compute, sidx, reinterpret_cast<float*>(b + L.dpart),
+                                                       counter, err);
+  CS_LAUNCHED();
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kCacheThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const int32_t* csidx = sidx;
+  const float2* no_drift = nullptr;
+  float* no_accum = nullptr;
+  uint8_t* no_u8 = nullptr;
+  int32_t* no_i32 = nullptr;
+  const uint8_t* no_force = nullptr;
+  unsigned* no_counter = nullptr;
+  if (target)
+    CS_CUDA(cudaLaunchKernelEx(&cfg, carry_skip_kernel<true, false>, x, x_ref, delta, no_accum, has_ref, N, D, nun, 0,
+                               tau, no_force, no_u8, no_i32, no_i32, csidx, no_drift, co, no_counter, h, t_next,
+                               target, spart, err));
+  else
+    CS_CUDA(cudaLaunchKernelEx(&cfg, carry_skip_kernel<false, false>, x, x_ref, delta, no_accum, has_ref, N, D, nun,
+                               0, tau, no_force, no_u8, no_i32, no_i32, csidx, no_drift, co, no_counter, h, t_next,
+                               (const float*)nullptr, (float*)nullptr, err));
+  CS_LAUNCHED();
+  return CS_OK;
+}
+
+cs_status carry_apply_tokens_run(float* x, float* x_ref, float* delta, float* accum, uint8_t* has_ref,
+                                 uint8_t* skip_mask, const float* hout, const int32_t* idx, int n_c, int N, int C,
+                                 int F, int H, int W, int step_k, float t_cur, float t_next, const float* target,
+                                 float* scores, const CarryState& cs, long long idx_limit, int* err,
+                                 cudaStream_t stream) {
+  const long long D = cs.D;
+  const int ntiles = F * (H / 2);
+  const StepLayout L = step_layout(cs.cap, D, cs.ntiles);
+  char* b = static_cast<char*>(cs.base);
+  const CarryOut co = carry_out(cs, L, step_k);
+  float* spart = reinterpret_cast<float*>(b + L.spart);
+  float* tpart = reinterpret_cast<float*>(b + L.tpart);
+  const float h = t_next - t_cur;
+  const size_t smem = (size_t)(W / 4) * (2 * C + 1) * sizeof(float4);
+  if (n_c > 0) {
+    const dim3 grid(ntiles, n_c);
+    if (target)
+      velocity_update_kernel<true, true><<<grid, kCacheThreads, smem, stream>>>(
+          hout, idx, C, F, H, W, x, x_ref, delta, accum, has_ref, skip_mask, h, t_next, target, tpart, co, idx_limit,
+          err);
+    else
+      velocity_update_kernel<false, true><<<grid, kCacheThreads, smem, stream>>>(
+          hout, idx, C, F, H, W, x, x_ref, delta, accum, has_ref, skip_mask, h, t_next, nullptr, nullptr, co,
+          idx_limit, err);
+    CS_LAUNCHED();
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.gridDim = dim3(n_c);
+    cfg.blockDim = dim3(kCacheThreads);
+    cfg.stream = stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    CS_CUDA(cudaLaunchKernelEx(&cfg, carry_rows_finalize_kernel, idx, ntiles, co, idx_limit, err));
+    CS_LAUNCHED();
+  }
+  if (target) {
+    score_finalize_split_kernel<<<(N + 3) / 4, 128, 0, stream>>>(spart, L.nun, tpart, ntiles, skip_mask, N, scores);
     CS_LAUNCHED();
   }
   return CS_OK;
@@ -1085,6 +1665,44 @@ extern "C" cs_status cs_cache_apply_tokens(float* x, float* x_ref, float* delta,
   const float* spart = workspace ? static_cast<const float*>(workspace) + (size_t)N * cache_chunks(D) * 2 : nullptr;
   return apply_tokens_run(x, x_ref, delta, accum, has_ref, skip_mask, hout, idx, n_c, N, C, F, H, W, t_cur, t_next,
                           target, scores, spart, tile_partials, (long long)N, err, stream);
+}
+
+extern "C" size_t cs_cache_step_bytes(int N, int C, int F, int H, int W) {
+  if (N <= 0 || !apply_tokens_supported(C, F, H, W)) return 0;
+  return carry_state_bytes(N, (long long)C * F * H * W, F * (H / 2));
+}
+
+extern "C" cs_status cs_cache_decide_skip_carry(float* x, const float* x_ref, const float* delta, float* accum,
+                                                uint8_t* has_ref, int N, int C, int F, int H, int W, int step_k,
+                                                int T, float t_cur, float t_next, float tau, int K_w, int K_c,
+                                                const uint8_t* force, uint8_t* skip_mask, int32_t* idx,
+                                                int32_t* n_compute, const float* target, int carried,
+                                                void* step_ws, int* err, cudaStream_t stream) {
+  CS_REQUIRE(N > 0 && N <= 4096, "cs_cache_decide_skip_carry: need 0 < N <= 4096 (N=%d)", N);
+  CS_REQUIRE(apply_tokens_supported(C, F, H, W), "cs_cache_decide_skip_carry: latent %dx%dx%dx%d unsupported", C, F,
+             H, W);
+  CS_REQUIRE(x && x_ref && delta && accum && has_ref && skip_mask && idx && n_compute && step_ws,
+             "cs_cache_decide_skip_carry: null pointer");
+  CS_REQUIRE(step_k >= 1 && step_k <= T, "cs_cache_decide_skip_carry: step %d outside 1..T=%d", step_k, T);
+  const CarryState cs{step_ws, N, (long long)C * F * H * W, F * (H / 2)};
+  return carry_decide_skip_run(x, x_ref, delta, accum, has_ref, N, step_k, T, t_cur, t_next, tau, K_w, K_c, force,
+                               skip_mask, idx, n_compute, target, carried != 0, cs, err, stream);
+}
+
+extern "C" cs_status cs_cache_apply_tokens_carry(float* x, float* x_ref, float* delta, float* accum,
+                                                 uint8_t* has_ref, uint8_t* skip_mask, const float* hout,
+                                                 const int32_t* idx, int n_c, int N, int C, int F, int H, int W,
+                                                 int step_k, float t_cur, float t_next, const float* target,
+                                                 float* scores, void* step_ws, int* err, cudaStream_t stream) {
+  CS_REQUIRE(N > 0 && N <= 4096 && n_c >= 0 && n_c <= N, "cs_cache_apply_tokens_carry: bad N=%d / n_c=%d", N, n_c);
+  CS_REQUIRE(apply_tokens_supported(C, F, H, W), "cs_cache_apply_tokens_carry: latent %dx%dx%dx%d unsupported", C,
+             F, H, W);
+  CS_REQUIRE(x && x_ref && delta && accum && has_ref && skip_mask && step_ws && (n_c == 0 || (hout && idx)),
+             "cs_cache_apply_tokens_carry: null pointer");
+  CS_REQUIRE(!target || scores, "cs_cache_apply_tokens_carry: scoring needs scores");
+  const CarryState cs{step_ws, N, (long long)C * F * H * W, F * (H / 2)};
+  return carry_apply_tokens_run(x, x_ref, delta, accum, has_ref, skip_mask, hout, idx, n_c, N, C, F, H, W, step_k,
+                                t_cur, t_next, target, scores, cs, N, err, stream);
 }
 
 extern "C" cs_status cs_cache_apply_computed(float* x, float* x_ref, float* delta, const float* v,

@@ -52,6 +52,31 @@ cs_status apply_tokens_run(float* x, float* x_ref, float* delta, float* accum, u
                            float t_cur, float t_next, const float* target, float* scores, const float* spart,
                            float* tpart, long long idx_limit, int* err, cudaStream_t stream);
 bool apply_tokens_supported(int C, int F, int H, int W);
+
+// The carried form of the step's cache work (the drift of the next step left by each
+// update): a step workspace of carry_state_bytes(cap, D, ntiles) bytes, zero-filled once,
+// holding `cap` candidate slots (ntiles = F*H/2).  carry_decide_skip_run takes the
+// decisions from the carried drift when `carried` (or inside the window, where none is
+// needed), else from a drift pass; it reports *n_compute = -1 and changes nothing when a
+// cached candidate carries no drift.  carry_apply_tokens_run is apply_tokens_run that
+// also leaves the computed candidates' drift for step_k + 1.
+struct CarryState {
+  void* base;
+  int cap;
+  long long D;
+  int ntiles;
+};
+size_t carry_state_bytes(int cap, long long D, int ntiles);
+cs_status carry_decide_skip_run(float* x, const float* x_ref, const float* delta, float* accum, uint8_t* has_ref,
+                                int N, int step_k, int T, float t_cur, float t_next, float tau, int K_w, int K_c,
+                                const uint8_t* force, uint8_t* skip_mask, int32_t* idx, int32_t* n_compute,
+                                const float* target, bool carried, const CarryState& cs, int* err,
+                                cudaStream_t stream);
+cs_status carry_apply_tokens_run(float* x, float* x_ref, float* delta, float* accum, uint8_t* has_ref,
+                                 uint8_t* skip_mask, const float* hout, const int32_t* idx, int n_c, int N, int C,
+                                 int F, int H, int W, int step_k, float t_cur, float t_next, const float* target,
+                                 float* scores, const CarryState& cs, long long idx_limit, int* err,
+                                 cudaStream_t stream);
 cs_status load_cache_kernels();
 
 }  // namespace cs

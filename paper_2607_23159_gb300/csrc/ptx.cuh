@@ -173,6 +173,14 @@ __device__ __forceinline__ void tma_reduce_add_2d(const void* map, const void* s
                "r"(x), "r"(y), "r"(smem_u32(src))
                : "memory");
 }
+// Contiguous global -> shared copy by the TMA unit (no tensor map): both addresses 16-byte
+// aligned, bytes a multiple of 16; completes `bytes` of the mbarrier's transaction count.
+__device__ __forceinline__ void bulk_load_1d(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(src), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 // At most one of this thread's bulk groups may still be reading its shared-memory source.
 __device__ __forceinline__ void bulk_wait_read_1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }

@@ -53,13 +53,16 @@ def _time_cold(fn, reps, warmup):
     return times[len(times) // 2]
 
 
-def cache_step(N, lat, skip_frac, reps=9, warmup=3, seed=0):
+def cache_step(N, lat, skip_frac, reps=9, warmup=3, seed=0, carried=True):
     """One free step's cache work for N candidates on a C x F x H x W latent, as the search
-    step runs it: cs_cache_decide_skip (drift, decision, skipped updates), then
-    cs_cache_apply_tokens for the computing candidates (head output in token layout).  The
-    round(N (1 - skip_frac)) candidates that compute are a seeded random subset.  Returns
-    (median ms of single calls after an L2-evicting write, algorithmic bytes, skipped):
-    16 D bytes per skipped candidate, 24 D per computed one."""
+    step runs it.  carried (the step's own form): cs_cache_decide_skip_carry with the drift
+    the previous step left (decisions, skipped updates and their next drift in one
+    launch), then cs_cache_apply_tokens_carry for the computing candidates (head output in
+    token layout); 16 D bytes per skipped candidate, 20 D per computed one.  Otherwise the
+    drift-pass form, cs_cache_decide_skip + cs_cache_apply_tokens (24 D per computed one).
+    The round(N (1 - skip_frac)) candidates that compute are a seeded random subset.
+    Returns (median ms of single calls after an L2-evicting write, algorithmic bytes,
+    skipped)."""
     import torch
     from paper_2607_23159_gb300 import binding as B
     dev = "cuda"
@@ -73,6 +76,7 @@ def cache_step(N, lat, skip_frac, reps=9, warmup=3, seed=0):
     st["delta"].normal_(generator=g)
     st["has_ref"].fill_(1)
     ws = torch.zeros(B.cache_workspace_bytes(N, D) // 4 + 1, device=dev)
+    sws = torch.zeros(B.cache_step_bytes(N, C_, F_, H_, W_) // 4 + 1, device=dev)
     skip = torch.zeros(N, dtype=torch.uint8, device=dev)
     idx = torch.zeros(N, dtype=torch.int32, device=dev)
     nc = torch.zeros(1, dtype=torch.int32, device=dev)
@@ -81,14 +85,26 @@ def cache_step(N, lat, skip_frac, reps=9, warmup=3, seed=0):
     force[torch.randperm(N, generator=g, device=dev)[:n_comp]] = 1
     hout = torch.randn(max(1, n_comp) * F_ * (H_ // 2) * (W_ // 2), 4 * C_, device=dev, generator=g)
     comp_idx = torch.nonzero(force).to(torch.int32).reshape(-1)
+    if carried:
+        # step 19 with the drift pass leaves every candidate's drift for step 20
+        B.cache_decide_skip_carry(st, lat, 19, 50, 0.62, 0.6, 0.1, 5, 5, skip, idx, nc, sws, carried=False,
+                                  force=force)
+        B.cache_apply_tokens_carry(st, skip, hout, comp_idx, n_comp, lat, 19, 0.62, 0.6, sws)
 
     def run():
-        B.cache_decide_skip(st["x"], st["x_ref"], st["delta"], st["accum"], st["has_ref"], 20, 50, 0.6, 0.58,
-                            0.1, 5, 5, skip, idx, nc, ws, force=force)
-        B.cache_apply_tokens(st, skip, hout, comp_idx, n_comp, C_, F_, H_, W_, 0.6, 0.58)
+        if carried:
+            B.cache_decide_skip_carry(st, lat, 20, 50, 0.6, 0.58, 0.1, 5, 5, skip, idx, nc, sws, carried=True,
+                                      force=force)
+            B.cache_apply_tokens_carry(st, skip, hout, comp_idx, n_comp, lat, 20, 0.6, 0.58, sws)
+        else:
+            B.cache_decide_skip(st["x"], st["x_ref"], st["delta"], st["accum"], st["has_ref"], 20, 50, 0.6, 0.58,
+                                0.1, 5, 5, skip, idx, nc, ws, force=force)
+            B.cache_apply_tokens(st, skip, hout, comp_idx, n_comp, C_, F_, H_, W_, 0.6, 0.58)
     ms = _time_cold(run, reps, warmup)
+    if carried:
+        assert int(nc[0]) == n_comp, "the carried decision did not run"
     n_skip = N - n_comp
-    return ms, (n_skip * 16.0 + n_comp * 24.0) * D, n_skip
+    return ms, (n_skip * 16.0 + n_comp * (20.0 if carried else 24.0)) * D, n_skip
 
 
 def main():
@@ -110,6 +126,8 @@ def main():
     ap.add_argument("--D", type=int, default=2096640)
     ap.add_argument("--skip-frac", type=float, default=1.0)
     ap.add_argument("--latent", default="16x21x60x104", help="C x F x H x W of the latent (cache-tokens)")
+    ap.add_argument("--drift-pass", action="store_true",
+                    help="cache-tokens: the drift-pass form instead of the carried drift the search step uses")
     ap.add_argument("--reps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=2)
     ap.add_argument("--torch", action="store_true", help="time the PyTorch comparator instead")
@@ -196,7 +214,7 @@ def main():
         N, D = a.N, a.D
         lat = [int(v) for v in a.latent.split("x")]
         if a.kernel == "cache-tokens":
-            ms, byts, n_skip = cache_step(N, lat, a.skip_frac, a.reps, a.warmup)
+            ms, byts, n_skip = cache_step(N, lat, a.skip_frac, a.reps, a.warmup, carried=not a.drift_pass)
             D = lat[0] * lat[1] * lat[2] * lat[3]
             out.update(shape=dict(N=N, D=D, skipped=n_skip), ms=ms, gbs=byts / (ms / 1e3) / 1e9)
             print(json.dumps(out), flush=True)
