@@ -710,6 +710,8 @@ constexpr int kUnitElems = 4096;
 constexpr int kSkipStages = 4;
 constexpr int kSkipStageFloats = 3 * kUnitElems;
 constexpr size_t kSkipRingBytes = (size_t)kSkipStages * kSkipStageFloats * sizeof(float);
+constexpr int kSkipThreads = kCacheThreads + 32;   // eight consumer warps and one producer warp
+constexpr int kClaim = 2;                          // units a producer claims at a time
 
 __host__ __device__ inline int carry_units(long long D) {
   long long u = (D + kUnitElems - 1) / kUnitElems;
@@ -720,44 +722,77 @@ __host__ inline size_t carry_skip_smem(int N) {
   return kSkipRingBytes + (size_t)(3 * N + 15) / 16 * 16;   // + skipped list (16-bit) and flags
 }
 
-// The skip update of cs_search_step with the carried drift, one CTA per SM.  Per skipped
-// candidate and unit: x_next = x + h (x + Delta) (Eq. skip + Eq. euler), written back, and
-// the unit's partial pair of the next step's drift, (x_next - x_ref)^2 and x_ref^2 (thread
-// sums, warp trees, then the eight warps in order); with a target, the unit's score
-// partial.  Thread 0 keeps the ring full (cp.async.bulk, one mbarrier per stage, waits
-// bounded); the units of the CTA's contiguous share of (skipped candidate, unit) items are
-// consumed in order.  When the CTA finishes its units of a candidate it counts them in;
-// the CTA that completes the candidate sums its unit pairs (warp 0, fixed order) into
-// carry.drift_out.
+// Fixed-order sum of a candidate's n partial pairs by one warp (lane l adds l, l + 32, ...,
+// then the shuffle tree): the carried value does not depend on which CTA completes it.
+__device__ __forceinline__ void carry_finalize_warp(const CarryOut& c, int i, int n, int lane) {
+  __threadfence();
+  const float2* pp = c.part + (long long)i * c.P;
+  float s0 = 0.f, s1 = 0.f;
+  for (int q = lane; q < n; q += 32) {
+    const float2 a = __ldcg(pp + q);
+    s0 += a.x;
+    s1 += a.y;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    s0 += __shfl_xor_sync(0xffffffffu, s0, o);
+    s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+  }
+  if (lane == 0) {
+    c.drift_out[i] = make_float2(s0, s1);
+    c.cnt[i] = 0u;
+  }
+}
+
+// The skip update of cs_search_step with the carried drift, one CTA per SM, warp
+// specialised.  Per skipped candidate and unit: x_next = x + h (x + Delta) (Eq. skip +
+// Eq. euler), written back, and the unit's partial pair of the next step's drift,
+// (x_next - x_ref)^2 and x_ref^2 (thread sums over the unit's float4s, warp trees, then
+// the eight warps in order); with a target, the unit's score partial.
+//  producer warp  claims units two at a time from a counter shared by the grid (claimed
+//                 one claim ahead), so that CTAs that are served faster take more units;
+//                 keeps the four-stage ring full (cp.async.bulk of x, Delta and x_ref, one
+//                 mbarrier per stage, a sentinel when the units run out); when the
+//                 consumers release a stage it adds the unit's eight warp pairs in order
+//                 and stores them.
+//  consumer warps wait for a stage, update the unit, leave their warp sums and release it.
+// Every wait is bounded.  Every CTA counts itself in on one arrival counter; the CTA that
+// arrives last (every unit pair is stored by then) resets it and the claim counter, and
+// its warps sum each skipped candidate's unit pairs in order into carry.drift_out:
 //  kDecide  every CTA takes the same decisions from the same inputs (decide_carried) and
-//           so knows the skipped list; every CTA counts itself in on one arrival counter,
-//           and the CTA that arrives last (after every CTA has read the state) writes
-//           accum, has_ref (3 for skipped candidates, whose new sums are complete), the
-//           skip mask and the list of computing candidates, and leaves the counter at
-//           zero.  A free step on which a cached candidate carries no drift changes
-//           nothing and reports *n_compute = -1: the caller then runs the drift pass.
+//           so knows the skipped list; the CTA that arrives last (after every CTA has read
+//           the state) also writes accum, has_ref (3 for skipped candidates), the skip
+//           mask and the list of computing candidates.  A free step on
+//           which a cached candidate carries no drift changes nothing and reports
+//           *n_compute = -1: the caller then runs the drift pass.
 //  !kDecide the decisions and the skipped list come from drift_decide_kernel (launched
-//           before this one with programmatic stream serialisation); the CTA completing a
-//           candidate sets its has_ref to 3.
+//           before this one with programmatic stream serialisation); the last CTA sets the
+//           skipped candidates' has_ref to 3.
 template <bool kScore, bool kDecide>
-__global__ void __launch_bounds__(kCacheThreads, 1) carry_skip_kernel(
+__global__ void __launch_bounds__(kSkipThreads, 1) carry_skip_kernel(
     float* __restrict__ x, const float* __restrict__ xr, const float* __restrict__ delta, float* __restrict__ accum,
     uint8_t* __restrict__ has_ref, int N, long long D, int nun, int wf, float tau, const uint8_t* __restrict__ force,
     uint8_t* __restrict__ skip_mask, int32_t* __restrict__ idx, int32_t* __restrict__ n_compute,
-    const int32_t* sidx_in, const float2* __restrict__ drift_in, CarryOut carry,
-    unsigned* __restrict__ counter, float h, float t_next, const float* __restrict__ target,
-    float* __restrict__ spart, int* err) {
+    const int32_t* sidx_in, const float2* __restrict__ drift_in, CarryOut carry, unsigned* __restrict__ counter,
+    unsigned* __restrict__ claim, float h, float t_next, const float* __restrict__ target, float* __restrict__ spart,
+    int* err) {
   constexpr int NV = kScore ? 3 : 2;
+  constexpr int S = kSkipStages;
   extern __shared__ __align__(128) uint8_t smem[];
   float* ring = reinterpret_cast<float*>(smem);
   uint16_t* s_list = reinterpret_cast<uint16_t*>(smem + kSkipRingBytes);
   uint8_t* s_flag = reinterpret_cast<uint8_t*>(s_list + N);
-  __shared__ uint64_t full[kSkipStages];
-  __shared__ float red[2][NV][kCacheWarps];
+  __shared__ uint64_t full[S], empty[S];
+  __shared__ int s_item[S];
+  __shared__ float red[S][NV][kCacheWarps];
   __shared__ int s_ns, s_bad, s_last, s_abort;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const bool producer = warp == kCacheWarps;
   if (threadIdx.x == 0) {
-    for (int q = 0; q < kSkipStages; ++q) mbar_init(&full[q], 1);
+    for (int q = 0; q < S; ++q) {
+      mbar_init(&full[q], 1);
+      mbar_init(&empty[q], kCacheWarps);
+    }
     fence_mbar_init();
     s_bad = 0;
     s_abort = 0;
@@ -765,7 +800,7 @@ __global__ void __launch_bounds__(kCacheThreads, 1) carry_skip_kernel(
   block_sync();
   int ns;
   if (kDecide) {
-    for (int i = threadIdx.x; i < N; i += kCacheThreads) {
+    for (int i = threadIdx.x; i < N; i += kSkipThreads) {
       float a;
       const uint8_t fl = decide_carried(i, wf, tau, has_ref, accum, drift_in, force, a);
       s_flag[i] = fl;
@@ -790,123 +825,125 @@ __global__ void __launch_bounds__(kCacheThreads, 1) carry_skip_kernel(
     // them through L2 (a read-only cached load could be placed before the wait)
     pdl_wait_primary();
     ns = __ldcg(sidx_in + N);
-    for (int q = threadIdx.x; q < ns; q += kCacheThreads) s_list[q] = (uint16_t)__ldcg(sidx_in + q);
+    for (int q = threadIdx.x; q < ns; q += kSkipThreads) s_list[q] = (uint16_t)__ldcg(sidx_in + q);
     block_sync();
   }
-  // this CTA's items: a balanced contiguous share of the (skipped candidate, unit) items
-  const long long items = (long long)ns * nun;
-  const int it0 = (int)(items * blockIdx.x / gridDim.x), it1 = (int)(items * (blockIdx.x + 1) / gridDim.x);
-  const int n_it = it1 - it0;
-  auto issue = [&](int k) {                       // thread 0: item k of this CTA into stage k % S
-    const int it = it0 + k, sq = it / nun, u = it - sq * nun, i = s_list[sq];
-    const long long lo = (long long)u * kUnitElems;
-    const uint32_t bytes = (uint32_t)(min((long long)kUnitElems, D - lo) * sizeof(float));
-    float* st = ring + (size_t)(k % kSkipStages) * kSkipStageFloats;
-    uint64_t* bar = &full[k % kSkipStages];
-    mbar_arrive_expect_tx(bar, 3 * bytes);
-    bulk_load_1d(st, x + (long long)i * D + lo, bytes, bar);
-    bulk_load_1d(st + kUnitElems, delta + (long long)i * D + lo, bytes, bar);
-    bulk_load_1d(st + 2 * kUnitElems, xr + (long long)i * D + lo, bytes, bar);
-  };
-  if (threadIdx.x == 0)
-    for (int k = 0; k < kSkipStages && k < n_it; ++k) issue(k);
-  int done_from = 0;                              // first item of the current candidate's run
-  int n_consumed = n_it;
-  for (int k = 0; k < n_it; ++k) {
-    const int sq = (it0 + k) / nun, u = it0 + k - sq * nun, i = s_list[sq];
-    if (!mbar_wait(&full[k % kSkipStages], (uint32_t)(k / kSkipStages) & 1u, (volatile int*)&s_abort, err)) {
-      n_consumed = k;
-      break;
-    }
-    const float* st = ring + (size_t)(k % kSkipStages) * kSkipStageFloats;
-    const float4* sx = reinterpret_cast<const float4*>(st);
-    const float4* sd = reinterpret_cast<const float4*>(st + kUnitElems);
-    const float4* sr = reinterpret_cast<const float4*>(st + 2 * kUnitElems);
-    const long long lo = (long long)u * kUnitElems;
-    const int n4 = (int)(min((long long)kUnitElems, D - lo) >> 2);
-    float4* xo = reinterpret_cast<float4*>(x + (long long)i * D + lo);
-    const float4* y4 = kScore ? reinterpret_cast<const float4*>(target + lo) : nullptr;
-    float acc[NV];
-#pragma unroll
-    for (int q = 0; q < NV; ++q) acc[q] = 0.f;
-#pragma unroll 4
-    for (int q = threadIdx.x; q < n4; q += kCacheThreads) {
-      const float4 xv = sx[q], dv = sd[q], rv = sr[q];
-      const float4 vu = make_float4(xv.x + dv.x, xv.y + dv.y, xv.z + dv.z, xv.w + dv.w);            // Eq. skip
-      const float4 xn = make_float4(xv.x + h * vu.x, xv.y + h * vu.y, xv.z + h * vu.z, xv.w + h * vu.w);  // Eq. euler
-      __stcs(xo + q, xn);
-      const float d0 = xn.x - rv.x, d1 = xn.y - rv.y, d2 = xn.z - rv.z, d3 = xn.w - rv.w;
-      acc[0] += d0 * d0 + d1 * d1 + d2 * d2 + d3 * d3;
-      acc[1] += rv.x * rv.x + rv.y * rv.y + rv.z * rv.z + rv.w * rv.w;
-      if (kScore) {
-        const float4 y = __ldg(y4 + q);
-        const float e0 = xn.x - t_next * vu.x - y.x, e1 = xn.y - t_next * vu.y - y.y;
-        const float e2 = xn.z - t_next * vu.z - y.z, e3 = xn.w - t_next * vu.w - y.w;
-        acc[2] += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
+  const int items = ns * nun;
+  volatile int* abort = &s_abort;
+  if (producer) {
+    // ---- producer warp: lane 0 claims and issues, the whole warp finalizes candidates
+    int next_claim = 0, cur = 0, left = 0, n_real = 0;
+    bool exhausted = false;
+    if (lane == 0 && items > 0) next_claim = (int)atomicAdd(claim, (unsigned)kClaim);
+    auto fill = [&](int j) {                       // lane 0: use j of stage j % S
+      const int st = j % S;
+      if (left == 0) {
+        cur = next_claim;
+        left = kClaim;
+        next_claim = (int)atomicAdd(claim, (unsigned)kClaim);   // needed one claim later
       }
-    }
-#pragma unroll
-    for (int q = 0; q < NV; ++q) {
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) acc[q] += __shfl_xor_sync(0xffffffffu, acc[q], o);
-    }
-    if (lane == 0) {
-#pragma unroll
-      for (int q = 0; q < NV; ++q) red[k & 1][q][warp] = acc[q];
-    }
-    block_sync();                                 // every thread is done with stage k % S
-    if (warp == 0) {
-      int fin = 0;
+      const int it = cur;
+      ++cur;
+      --left;
+      if (it >= items) {
+        s_item[st] = -1;
+        mbar_arrive(&full[st]);
+        exhausted = true;
+        return;
+      }
+      const int sq = it / nun, u = it - sq * nun, i = s_list[sq];
+      const long long lo = (long long)u * kUnitElems;
+      const uint32_t bytes = (uint32_t)(min((long long)kUnitElems, D - lo) * sizeof(float));
+      float* dst = ring + (size_t)st * kSkipStageFloats;
+      s_item[st] = it;
+      mbar_arrive_expect_tx(&full[st], 3 * bytes);
+      bulk_load_1d(dst, x + (long long)i * D + lo, bytes, &full[st]);
+      bulk_load_1d(dst + kUnitElems, delta + (long long)i * D + lo, bytes, &full[st]);
+      bulk_load_1d(dst + 2 * kUnitElems, xr + (long long)i * D + lo, bytes, &full[st]);
+      ++n_real;
+    };
+    if (lane == 0 && items > 0)
+      for (int j = 0; j < S && !exhausted; ++j) fill(j);
+    n_real = __shfl_sync(0xffffffffu, n_real, 0);
+    for (int j = 0; j < n_real; ++j) {
+      const int st = j % S;
+      if (!mbar_wait(&empty[st], (uint32_t)(j / S) & 1u, abort, err)) break;   // the consumers are done with use j
       if (lane == 0) {
+        const int it = s_item[st], sq = it / nun, u = it - sq * nun, i = s_list[sq];
         float p[NV];
 #pragma unroll
         for (int q = 0; q < NV; ++q) {
           p[q] = 0.f;
 #pragma unroll
-          for (int w = 0; w < kCacheWarps; ++w) p[q] += red[k & 1][q][w];
+          for (int w = 0; w < kCacheWarps; ++w) p[q] += red[st][q][w];
         }
         carry.part[(long long)i * carry.P + u] = make_float2(p[0], p[1]);
         if (kScore) spart[(long long)i * nun + u] = p[NV - 1];
-        if (k + kSkipStages < n_it) issue(k + kSkipStages);
-        const bool last_of_run = k + 1 == n_it || (it0 + k + 1) / nun != sq;
-        if (last_of_run) {
-          const unsigned run = (unsigned)(k - done_from + 1);
-          __threadfence();
-          fin = atomicAdd(carry.cnt + i, run) + run == (unsigned)nun;
-        }
+        if (!exhausted) fill(j + S);
       }
-      fin = __shfl_sync(0xffffffffu, fin, 0);
-      if (fin) {   // the candidate is complete: warp 0 sums its unit pairs in a fixed order
-        __threadfence();
-        const float2* pp = carry.part + (long long)i * carry.P;
-        float s0 = 0.f, s1 = 0.f;
-        for (int q = lane; q < nun; q += 32) {
-          const float2 a = __ldcg(pp + q);
-          s0 += a.x;
-          s1 += a.y;
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-          s0 += __shfl_xor_sync(0xffffffffu, s0, o);
-          s1 += __shfl_xor_sync(0xffffffffu, s1, o);
-        }
-        if (lane == 0) {
-          carry.drift_out[i] = make_float2(s0, s1);
-          carry.cnt[i] = 0u;
-          if (!kDecide) has_ref[i] = 3;
-        }
-      }
+      n_real = __shfl_sync(0xffffffffu, n_real, 0);
     }
-    if (k + 1 < n_it && (it0 + k + 1) / nun != sq) done_from = k + 1;
+    if (*abort && lane == 0) {
+      // a wait ran out: let every copy this CTA issued land before its memory goes
+      for (int j = 0; j < n_real; ++j) mbar_wait_teardown(&full[j % S], (uint32_t)(j / S) & 1u);
+    }
+    if (lane == 0 && items > 0) {
+      // the claim made ahead must be performed before this CTA arrives (the last CTA to
+      // arrive resets the counter): wait for its value
+      if (next_claim < 0) record_error(err, CS_ERR_ARG);
+      __threadfence();
+    }
+  } else if (items > 0) {
+    // ---- consumer warps
+    for (int j = 0;; ++j) {
+      const int st = j % S;
+      if (!mbar_wait(&full[st], (uint32_t)(j / S) & 1u, abort, err)) break;
+      const int it = s_item[st];
+      if (it < 0) break;
+      const int sq = it / nun, u = it - sq * nun, i = s_list[sq];
+      const float* sb = ring + (size_t)st * kSkipStageFloats;
+      const float4* sx = reinterpret_cast<const float4*>(sb);
+      const float4* sd = reinterpret_cast<const float4*>(sb + kUnitElems);
+      const float4* sr = reinterpret_cast<const float4*>(sb + 2 * kUnitElems);
+      const long long lo = (long long)u * kUnitElems;
+      const int n4 = (int)(min((long long)kUnitElems, D - lo) >> 2);
+      float4* xo = reinterpret_cast<float4*>(x + (long long)i * D + lo);
+      const float4* y4 = kScore ? reinterpret_cast<const float4*>(target + lo) : nullptr;
+      float acc[NV];
+#pragma unroll
+      for (int q = 0; q < NV; ++q) acc[q] = 0.f;
+#pragma unroll 4
+      for (int q = threadIdx.x; q < n4; q += kCacheThreads) {
+        const float4 xv = sx[q], dv = sd[q], rv = sr[q];
+        const float4 vu = make_float4(xv.x + dv.x, xv.y + dv.y, xv.z + dv.z, xv.w + dv.w);            // Eq. skip
+        const float4 xn = make_float4(xv.x + h * vu.x, xv.y + h * vu.y, xv.z + h * vu.z, xv.w + h * vu.w);  // Eq. euler
+        __stcs(xo + q, xn);
+        const float d0 = xn.x - rv.x, d1 = xn.y - rv.y, d2 = xn.z - rv.z, d3 = xn.w - rv.w;
+        acc[0] += d0 * d0 + d1 * d1 + d2 * d2 + d3 * d3;
+        acc[1] += rv.x * rv.x + rv.y * rv.y + rv.z * rv.z + rv.w * rv.w;
+        if (kScore) {
+          const float4 y = __ldg(y4 + q);
+          const float e0 = xn.x - t_next * vu.x - y.x, e1 = xn.y - t_next * vu.y - y.y;
+          const float e2 = xn.z - t_next * vu.z - y.z, e3 = xn.w - t_next * vu.w - y.w;
+          acc[2] += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < NV; ++q) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) acc[q] += __shfl_xor_sync(0xffffffffu, acc[q], o);
+      }
+      if (lane == 0) {
+#pragma unroll
+        for (int q = 0; q < NV; ++q) red[st][q][warp] = acc[q];
+        mbar_arrive(&empty[st]);
+      }
+      __syncwarp();
+    }
   }
-  if (s_abort && threadIdx.x == 0) {
-    // a wait ran out: let the copies already issued (items n_consumed .. n_consumed + S - 1
-    // at most) land before the CTA's memory goes
-    for (int k = n_consumed; k < n_it && k < n_consumed + kSkipStages; ++k)
-      mbar_wait_teardown(&full[k % kSkipStages], (uint32_t)(k / kSkipStages) & 1u);
-  }
-  if (!kDecide) return;
-  // arrival: the CTA that arrives last (every CTA has read the state by then) writes it
+  block_sync();
+  // arrival: the CTA that arrives last (every CTA has read the state and claimed its last
+  // unit by then) resets both counters and, deciding, writes the state
   if (threadIdx.x == 0) {
     __threadfence();
     s_last = atomicAdd(counter, 1u) == gridDim.x - 1;
@@ -914,14 +951,21 @@ __global__ void __launch_bounds__(kCacheThreads, 1) carry_skip_kernel(
   block_sync();
   if (!s_last) return;
   __threadfence();
+  if (threadIdx.x == 0) {
+    *claim = 0u;
+    *counter = 0u;
+  }
   if (s_bad) {
-    if (threadIdx.x == 0) {
-      *n_compute = -1;
-      *counter = 0u;
-    }
+    if (threadIdx.x == 0) *n_compute = -1;
     return;
   }
-  for (int i = threadIdx.x; i < N; i += kCacheThreads) {
+  // every unit pair is stored: one warp per skipped candidate sums them in order
+  for (int q = warp; q < ns; q += kSkipThreads / 32) {
+    carry_finalize_warp(carry, s_list[q], nun, lane);
+    if (!kDecide && lane == 0) has_ref[s_list[q]] = 3;
+  }
+  if (!kDecide) return;
+  for (int i = threadIdx.x; i < N; i += kSkipThreads) {
     float a;
     const uint8_t fl = decide_carried(i, wf, tau, has_ref, accum, drift_in, force, a);
     const bool compute = fl & kFlCompute;
@@ -942,10 +986,7 @@ __global__ void __launch_bounds__(kCacheThreads, 1) carry_skip_kernel(
       if (comp) idx[nc + __popc(b & ((1u << lane) - 1u))] = k;
       nc += __popc(b);
     }
-    if (lane == 0) {
-      *n_compute = nc;
-      *counter = 0u;
-    }
+    if (lane == 0) *n_compute = nc;
   }
 }
 
@@ -1064,13 +1105,13 @@ __global__ void __launch_bounds__(kCacheThreads) velocity_update_kernel(
   float acc[NV];
 #pragma unroll
   for (int q = 0; q < NV; ++q) acc[q] = 0.f;
-  auto offset = [&](int q, int& cp, int& w4) {
-    w4 = q % W4;
-    cp = q / W4;                                  // cp = 2c + (h & 1)
-    return (((long long)(cp >> 1) * F + f) * H + 2 * hh + (cp & 1)) * W + 4 * w4;
+  // element offset of update item q inside the candidate's latent (D < 2^31 elements)
+  auto offset = [&](int q) {
+    const int w4 = q % W4, cp = q / W4;           // cp = 2c + (h & 1)
+    return (((cp >> 1) * F + f) * H + 2 * hh + (cp & 1)) * W + 4 * w4;
   };
-  auto update = [&](long long e, int cp, int w4, float4 xv) {
-    const float4 vu = s_v[w4 * S + cp];
+  auto update = [&](int q, int e, float4 xv) {
+    const float4 vu = s_v[(q % W4) * S + q / W4];
     __stcs(reinterpret_cast<float4*>(di + e), make_float4(vu.x - xv.x, vu.y - xv.y, vu.z - xv.z, vu.w - xv.w));
     __stcs(reinterpret_cast<float4*>(ri + e), xv);
     const float4 xn = make_float4(xv.x + h * vu.x, xv.y + h * vu.y, xv.z + h * vu.z, xv.w + h * vu.w);
@@ -1090,24 +1131,18 @@ __global__ void __launch_bounds__(kCacheThreads) velocity_update_kernel(
   const int nu = 2 * C * W4;
   {
     float4 xv[kVelUnroll];
-    long long e[kVelUnroll];
-    int cp[kVelUnroll], w4[kVelUnroll];
 #pragma unroll
     for (int u = 0; u < kVelUnroll; ++u) {
       const int q = threadIdx.x + u * kCacheThreads;
-      if (q < nu) {
-        e[u] = offset(q, cp[u], w4[u]);
-        xv[u] = __ldcs(reinterpret_cast<const float4*>(xi + e[u]));
-      }
+      if (q < nu) xv[u] = __ldcs(reinterpret_cast<const float4*>(xi + offset(q)));
     }
 #pragma unroll
-    for (int u = 0; u < kVelUnroll; ++u)
-      if (threadIdx.x + u * kCacheThreads < nu) update(e[u], cp[u], w4[u], xv[u]);
-    for (int q = threadIdx.x + kVelUnroll * kCacheThreads; q < nu; q += kCacheThreads) {
-      int c2, w2;
-      const long long e2 = offset(q, c2, w2);
-      update(e2, c2, w2, __ldcs(reinterpret_cast<const float4*>(xi + e2)));
+    for (int u = 0; u < kVelUnroll; ++u) {
+      const int q = threadIdx.x + u * kCacheThreads;
+      if (q < nu) update(q, offset(q), xv[u]);
     }
+    for (int q = threadIdx.x + kVelUnroll * kCacheThreads; q < nu; q += kCacheThreads)
+      update(q, offset(q), __ldcs(reinterpret_cast<const float4*>(xi + offset(q))));
   }
   if (kScore || kCarry) {
     block_sum<NV>(acc, red);
@@ -1441,13 +1476,13 @@ cs_status apply_tokens_run(float* x, float* x_ref, float* delta, float* accum, u
 
 // ------------------------------------------------------------ carried form ----
 // Step workspace of the carried form for `cap` candidate slots, each part at a 256-byte
-// boundary: arrival counter; skipped list [cap + 1]; completion counts [cap]; carried
+// boundary: arrival counter; unit claim counter; skipped list [cap + 1]; completion counts [cap]; carried
 // sums [2][cap] (float2, by the parity of the step that reads them); partial pairs
 // [cap][max(units, F*H/2)] (float2; units of 4096 elements); drift-pass partials
 // [cap][nch][2]; skipped candidates' score partials [cap][units]; computed candidates'
 // score partials [cap][F*H/2].
 struct StepLayout {
-  size_t counter, sidx, cnt, drift, part, dpart, spart, tpart, total;
+  size_t counter, claim, sidx, cnt, drift, part, dpart, spart, tpart, total;
   int nch, nun, P;
 };
 
@@ -1464,6 +1499,7 @@ static StepLayout step_layout(int cap, long long D, int ntiles) {
   L.nun = carry_units(D);
   L.P = L.nun > ntiles ? L.nun : ntiles;
   L.counter = take(sizeof(unsigned));
+  L.claim = take(sizeof(unsigned));
   L.sidx = take((size_t)(cap + 1) * sizeof(int32_t));
   L.cnt = take((size_t)cap * sizeof(unsigned));
   L.drift = take((size_t)2 * cap * sizeof(float2));
@@ -1516,6 +1552,7 @@ cs_status carry_decide_skip_run(float* x, const float* x_ref, const float* delta
   const StepLayout L = step_layout(cs.cap, D, cs.ntiles);
   char* b = static_cast<char*>(cs.base);
   unsigned* counter = reinterpret_cast<unsigned*>(b + L.counter);
+  unsigned* claim = reinterpret_cast<unsigned*>(b + L.claim);
   int32_t* sidx = reinterpret_cast<int32_t*>(b + L.sidx);
   const CarryOut co = carry_out(cs, L, step_k);
   const float2* din = reinterpret_cast<const float2*>(b + L.drift) + (size_t)(step_k & 1) * cs.cap;
@@ -1529,13 +1566,13 @@ cs_status carry_decide_skip_run(float* x, const float* x_ref, const float* delta
   if (carried || wf) {
     // decisions from the carried drift (none is needed inside the window): one launch
     if (target)
-      carry_skip_kernel<true, true><<<grid, kCacheThreads, smem, stream>>>(
+      carry_skip_kernel<true, true><<<grid, kSkipThreads, smem, stream>>>(
           x, x_ref, delta, accum, has_ref, N, D, nun, wf, tau, force, skip_mask, idx, n_compute, nullptr, din, co,
-          counter, h, t_next, target, spart, err);
+          counter, claim, h, t_next, target, spart, err);
     else
-      carry_skip_kernel<false, true><<<grid, kCacheThreads, smem, stream>>>(
+      carry_skip_kernel<false, true><<<grid, kSkipThreads, smem, stream>>>(
           x, x_ref, delta, accum, has_ref, N, D, nun, wf, tau, force, skip_mask, idx, n_compute, nullptr, din, co,
-          counter, h, t_next, nullptr, nullptr, err);
+          counter, claim, h, t_next, nullptr, nullptr, err);
     CS_LAUNCHED();
     return CS_OK;
   }
@@ -1552,7 +1589,7 @@ cs_status carry_decide_skip_run(float* x, const float* x_ref, const float* delta
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(kCacheThreads);
+  cfg.blockDim = dim3(kSkipThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cfg.attrs = attr;
@@ -1563,15 +1600,14 @@ cs_status carry_decide_skip_run(float* x, const float* x_ref, const float* delta
   uint8_t* no_u8 = nullptr;
   int32_t* no_i32 = nullptr;
   const uint8_t* no_force = nullptr;
-  unsigned* no_counter = nullptr;
   if (target)
     CS_CUDA(cudaLaunchKernelEx(&cfg, carry_skip_kernel<true, false>, x, x_ref, delta, no_accum, has_ref, N, D, nun, 0,
-                               tau, no_force, no_u8, no_i32, no_i32, csidx, no_drift, co, no_counter, h, t_next,
+                               tau, no_force, no_u8, no_i32, no_i32, csidx, no_drift, co, counter, claim, h, t_next,
                                target, spart, err));
   else
     CS_CUDA(cudaLaunchKernelEx(&cfg, carry_skip_kernel<false, false>, x, x_ref, delta, no_accum, has_ref, N, D, nun,
-                               0, tau, no_force, no_u8, no_i32, no_i32, csidx, no_drift, co, no_counter, h, t_next,
-                               (const float*)nullptr, (float*)nullptr, err));
+                               0, tau, no_force, no_u8, no_i32, no_i32, csidx, no_drift, co, counter, claim, h,
+                               t_next, (const float*)nullptr, (float*)nullptr, err));
   CS_LAUNCHED();
   return CS_OK;
 }
