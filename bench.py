@@ -449,8 +449,10 @@ def run_ours(args, cfg):
         from paper_2607_23159_gb300 import kernel_bench as KB
         hbm = measured_peaks().get("hbm_gbs") or 6800.0
         cases = []
-        for n_c, lat, sf in ((16, (16, 21, 60, 104), 1.0), (16, (16, 21, 60, 104), 0.5), (32, (16, 9, 30, 52), 1.0),
-                             (32, (16, 9, 30, 52), 0.5), (N, (m.C, m.F, m.H, m.W), 1.0), (N, (m.C, m.F, m.H, m.W), 0.5)):
+        sh = synth.WAN_1_3B_SHORT
+        ls = (sh.C, sh.F, sh.H, sh.W)
+        for n_c, lat, sf in ((16, (16, 21, 60, 104), 1.0), (16, (16, 21, 60, 104), 0.5), (32, ls, 1.0),
+                             (32, ls, 0.5), (N, (m.C, m.F, m.H, m.W), 1.0), (N, (m.C, m.F, m.H, m.W), 0.5)):
             c_ms, c_bytes, c_skip = KB.cache_step(n_c, lat, sf)
             gbs = c_bytes / (c_ms / 1e3) / 1e9
             cases.append({"N": n_c, "latent": "x".join(map(str, lat)), "skipped": c_skip, "us": c_ms * 1e3,
