@@ -5,6 +5,10 @@
 //           block turns them into a += drift, the skip decision and the compaction list.
 //  apply    Eq. delta / Eq. skip fused with Eq. euler (and, optionally, the x0-estimate
 //           score) in one pass over the candidate's latent.
+//  carry    the form cs_search_step runs: every update also leaves the next step's two
+//           drift sums (the values are in its registers), so a step decides from them
+//           without reading x or x_ref, and the skipped candidates' update (fed by TMA
+//           bulk copies) is the one pass over their state.
 //  score    -||x - y*||_2 (the verifier stand-in of Algorithm 1).
 //  topk     rank-by-counting selection, deterministic tie-break.
 //  refill   beam refill (state copy of survivors + seeded perturbation of children).
@@ -638,13 +642,13 @@ __global__ void __launch_bounds__(kCacheThreads, 4) skip_update_kernel(
 // has_ref = 3 (bit 1 set) marks a candidate whose carried sums belong to its current x
 // and x_ref; every other writer of the state leaves has_ref = 1.
 //
-// The partial pairs of a candidate are summed by whichever CTA completes its last chunk
-// or token row (per-candidate completion counter, left at zero), in a fixed order that
-// does not depend on that CTA, so the carried value depends on the candidate alone.
+// The partial pairs of a candidate (one per 4096-element unit of a skipped candidate, one
+// per token row of a computed one) are summed once every pair is stored, in a fixed order
+// that does not depend on which CTA sums them, so the carried value depends on the
+// candidate alone.
 struct CarryOut {
-  float2* part;        // [cap][P] partial pairs of the candidate's chunk warps or token rows
+  float2* part;        // [cap][P] partial pairs of the candidate's units or token rows
   int P;
-  unsigned* cnt;       // [cap] completion counts (zero between calls)
   float2* drift_out;   // [cap] (sum (x_next - x_ref)^2, sum x_ref^2) for the next step
 };
 
@@ -658,10 +662,7 @@ __device__ __forceinline__ void carry_finalize(const CarryOut& c, int i, int n, 
     v[1] += a.y;
   }
   block_sum<2>(v, red);
-  if (threadIdx.x == 0) {
-    c.drift_out[i] = make_float2(v[0], v[1]);
-    c.cnt[i] = 0u;
-  }
+  if (threadIdx.x == 0) c.drift_out[i] = make_float2(v[0], v[1]);
   block_sync();
 }
 
@@ -723,7 +724,7 @@ __host__ inline size_t carry_skip_smem(int N) {
 }
 
 // Fixed-order sum of a candidate's n partial pairs by one warp (lane l adds l, l + 32, ...,
-// then the shuffle tree): the carried value does not depend on which CTA completes it.
+// then the shuffle tree): the carried value does not depend on which CTA sums it.
 __device__ __forceinline__ void carry_finalize_warp(const CarryOut& c, int i, int n, int lane) {
   __threadfence();
   const float2* pp = c.part + (long long)i * c.P;
@@ -738,10 +739,7 @@ __device__ __forceinline__ void carry_finalize_warp(const CarryOut& c, int i, in
     s0 += __shfl_xor_sync(0xffffffffu, s0, o);
     s1 += __shfl_xor_sync(0xffffffffu, s1, o);
   }
-  if (lane == 0) {
-    c.drift_out[i] = make_float2(s0, s1);
-    c.cnt[i] = 0u;
-  }
+  if (lane == 0) c.drift_out[i] = make_float2(s0, s1);
 }
 
 // The skip update of cs_search_step with the carried drift, one CTA per SM, warp
@@ -1476,13 +1474,13 @@ cs_status apply_tokens_run(float* x, float* x_ref, float* delta, float* accum, u
 
 // ------------------------------------------------------------ carried form ----
 // Step workspace of the carried form for `cap` candidate slots, each part at a 256-byte
-// boundary: arrival counter; unit claim counter; skipped list [cap + 1]; completion counts [cap]; carried
+// boundary: arrival counter; unit claim counter; skipped list [cap + 1]; carried
 // sums [2][cap] (float2, by the parity of the step that reads them); partial pairs
 // [cap][max(units, F*H/2)] (float2; units of 4096 elements); drift-pass partials
 // [cap][nch][2]; skipped candidates' score partials [cap][units]; computed candidates'
 // score partials [cap][F*H/2].
 struct StepLayout {
-  size_t counter, claim, sidx, cnt, drift, part, dpart, spart, tpart, total;
+  size_t counter, claim, sidx, drift, part, dpart, spart, tpart, total;
   int nch, nun, P;
 };
 
@@ -1501,7 +1499,6 @@ static StepLayout step_layout(int cap, long long D, int ntiles) {
   L.counter = take(sizeof(unsigned));
   L.claim = take(sizeof(unsigned));
   L.sidx = take((size_t)(cap + 1) * sizeof(int32_t));
-  L.cnt = take((size_t)cap * sizeof(unsigned));
   L.drift = take((size_t)2 * cap * sizeof(float2));
   L.part = take((size_t)cap * L.P * sizeof(float2));
   L.dpart = take((size_t)cap * L.nch * 2 * sizeof(float));
@@ -1515,7 +1512,7 @@ size_t carry_state_bytes(int cap, long long D, int ntiles) { return step_layout(
 
 static CarryOut carry_out(const CarryState& cs, const StepLayout& L, int step_k) {
   char* b = static_cast<char*>(cs.base);
-  return CarryOut{reinterpret_cast<float2*>(b + L.part), L.P, reinterpret_cast<unsigned*>(b + L.cnt),
+  return CarryOut{reinterpret_cast<float2*>(b + L.part), L.P,
                   reinterpret_cast<float2*>(b + L.drift) + (size_t)((step_k + 1) & 1) * cs.cap};
 }
 

@@ -133,3 +133,25 @@ def test_product_path_has_no_fallback():
             "    print('refused:', e)\n")
     out = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, cwd=ROOT, timeout=120)
     assert out.returncode == 0 and out.stdout.startswith("refused:") and "build" in out.stdout, out.stdout + out.stderr
+
+
+def test_step_workspace_size_of_the_carried_form(b):
+    """cs_cache_step_bytes: 0 for latents the token-layout update does not handle (odd H,
+    W not a multiple of 4) and for N <= 0; otherwise it covers at least the carried sums
+    (two float2 per candidate, by step parity), the unit and token-row partial pairs and
+    the drift-pass partials, and grows with N."""
+    from paper_2607_23159_gb300 import synth
+    assert b.cache_step_bytes(4, 16, 21, 60, 102) == 0
+    assert b.cache_step_bytes(4, 16, 21, 59, 104) == 0
+    assert b.cache_step_bytes(0, 16, 21, 60, 104) == 0
+    m = synth.WAN_1_3B
+    units = -(-m.D // 4096)
+    rows = m.F * m.H // 2
+    chunks = -(-m.D // 8192)
+    for N in (1, 4, 16):
+        got = b.cache_step_bytes(N, m.C, m.F, m.H, m.W)
+        assert got % 256 == 0
+        assert got >= N * (2 * 8 + max(units, rows) * 8 + chunks * 8 + units * 4 + rows * 4)
+    assert b.cache_step_bytes(16, m.C, m.F, m.H, m.W) > b.cache_step_bytes(4, m.C, m.F, m.H, m.W)
+    t = synth.TINY
+    assert b.cache_step_bytes(4, t.C, t.F, t.H, t.W) > 0

@@ -31,7 +31,7 @@ def test_bench_line_on_the_tiny_workload():
     assert f["T"] == d["config"]["T"] and f["value"] > 0 and 0 < f["computed_fraction"] <= 1
     assert f["cache_update"]["launches"] > 0 and f["unit"] == d["unit"]
     cases = d["cache_alone"]["cases"]
-    assert [(c["N"], c["latent"]) for c in cases[:4]] == [(16, "16x21x60x104")] * 2 + [(32, "16x9x30x52")] * 2
+    assert [(c["N"], c["latent"]) for c in cases[:4]] == [(16, "16x21x60x104")] * 2 + [(32, "16x9x60x104")] * 2
     assert all(c["gbs"] > 0 and 0 <= c["skipped"] <= c["N"] for c in cases)
 
 
