@@ -676,16 +676,19 @@ constexpr uint8_t kFlCompute = 1, kFlNonFinite = 2, kFlArg = 4, kFlBad = 8;
 __device__ __forceinline__ uint8_t decide_carried(int i, int wf, float tau, const uint8_t* __restrict__ has_ref,
                                                   const float* __restrict__ accum, const float2* __restrict__ drift_in,
                                                   const uint8_t* __restrict__ force, float& a) {
+  // every input loaded before the first use (one round trip, not one per branch)
   const uint8_t hr = has_ref[i];
+  const float a0 = accum[i];
+  const float2 s2 = drift_in[i];
+  const uint8_t fi = force ? force[i] : 0;
   const bool had = hr != 0;
   bool compute = true;
   uint8_t fl = 0;
-  a = accum[i];
+  a = a0;
   if (!wf && had) {
     if (!(hr & 2)) {
       fl |= kFlBad;
     } else {
-      const float2 s2 = drift_in[i];
       const float drift = drift_of(s2.x, s2.y);
       if (!isfinite(drift)) {
         fl |= kFlNonFinite;
@@ -696,7 +699,7 @@ __device__ __forceinline__ uint8_t decide_carried(int i, int wf, float tau, cons
     }
   }
   if (force) {
-    const bool f = force[i] != 0;
+    const bool f = fi != 0;
     if (!f && !had) fl |= kFlArg;
     else compute = f;
   }
@@ -729,10 +732,19 @@ __device__ __forceinline__ void carry_finalize_warp(const CarryOut& c, int i, in
   __threadfence();
   const float2* pp = c.part + (long long)i * c.P;
   float s0 = 0.f, s1 = 0.f;
-  for (int q = lane; q < n; q += 32) {
-    const float2 a = __ldcg(pp + q);
-    s0 += a.x;
-    s1 += a.y;
+  constexpr int kU = 16;                 // loads in flight per lane before the adds
+  for (int base = 0; base < n; base += 32 * kU) {
+    float2 v[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int q = base + lane + 32 * u;
+      v[u] = q < n ? __ldcg(pp + q) : make_float2(0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {       // the same order as one pair at a time (adding 0 changes nothing)
+      s0 += v[u].x;
+      s1 += v[u].y;
+    }
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -747,8 +759,9 @@ __device__ __forceinline__ void carry_finalize_warp(const CarryOut& c, int i, in
 // Eq. euler), written back, and the unit's partial pair of the next step's drift,
 // (x_next - x_ref)^2 and x_ref^2 (thread sums over the unit's float4s, warp trees, then
 // the eight warps in order); with a target, the unit's score partial.
-//  producer warp  claims units two at a time from a counter shared by the grid (claimed
-//                 one claim ahead), so that CTAs that are served faster take more units;
+//  producer warp  claims units from a counter shared by the grid (a full ring at kernel
+//                 start, while the decisions are taken, then two at a time, one claim
+//                 ahead), so that CTAs that are served faster take more units;
 //                 keeps the four-stage ring full (cp.async.bulk of x, Delta and x_ref, one
 //                 mbarrier per stage, a sentinel when the units run out); when the
 //                 consumers release a stage it adds the unit's eight warp pairs in order
@@ -786,6 +799,13 @@ __global__ void __launch_bounds__(kSkipThreads, 1) carry_skip_kernel(
   __shared__ int s_ns, s_bad, s_last, s_abort;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const bool producer = warp == kCacheWarps;
+  // the producer's first claims (a full ring, then the next claim) go out now, so that their
+  // round trips overlap the decisions; claims past the last item become sentinels
+  unsigned first_claim = 0, next_claim = 0;
+  if (producer && lane == 0) {
+    first_claim = atomicAdd(claim, (unsigned)S);
+    next_claim = atomicAdd(claim, (unsigned)kClaim);
+  }
   if (threadIdx.x == 0) {
     for (int q = 0; q < S; ++q) {
       mbar_init(&full[q], 1);
@@ -830,15 +850,14 @@ __global__ void __launch_bounds__(kSkipThreads, 1) carry_skip_kernel(
   volatile int* abort = &s_abort;
   if (producer) {
     // ---- producer warp: lane 0 claims and issues, the whole warp finalizes candidates
-    int next_claim = 0, cur = 0, left = 0, n_real = 0;
+    int cur = (int)first_claim, left = S, n_real = 0;
     bool exhausted = false;
-    if (lane == 0 && items > 0) next_claim = (int)atomicAdd(claim, (unsigned)kClaim);
     auto fill = [&](int j) {                       // lane 0: use j of stage j % S
       const int st = j % S;
       if (left == 0) {
-        cur = next_claim;
+        cur = (int)next_claim;
         left = kClaim;
-        next_claim = (int)atomicAdd(claim, (unsigned)kClaim);   // needed one claim later
+        next_claim = atomicAdd(claim, (unsigned)kClaim);   // needed one claim later
       }
       const int it = cur;
       ++cur;
@@ -885,10 +904,10 @@ __global__ void __launch_bounds__(kSkipThreads, 1) carry_skip_kernel(
       // a wait ran out: let every copy this CTA issued land before its memory goes
       for (int j = 0; j < n_real; ++j) mbar_wait_teardown(&full[j % S], (uint32_t)(j / S) & 1u);
     }
-    if (lane == 0 && items > 0) {
-      // the claim made ahead must be performed before this CTA arrives (the last CTA to
-      // arrive resets the counter): wait for its value
-      if (next_claim < 0) record_error(err, CS_ERR_ARG);
+    if (lane == 0) {
+      // the claims made ahead must be performed before this CTA arrives (the last CTA to
+      // arrive resets the counter): wait for their values
+      if ((int)(first_claim | next_claim) < 0) record_error(err, CS_ERR_ARG);
       __threadfence();
     }
   } else if (items > 0) {
@@ -962,29 +981,30 @@ __global__ void __launch_bounds__(kSkipThreads, 1) carry_skip_kernel(
     carry_finalize_warp(carry, s_list[q], nun, lane);
     if (!kDecide && lane == 0) has_ref[s_list[q]] = 3;
   }
-  if (!kDecide) return;
-  for (int i = threadIdx.x; i < N; i += kSkipThreads) {
-    float a;
-    const uint8_t fl = decide_carried(i, wf, tau, has_ref, accum, drift_in, force, a);
-    const bool compute = fl & kFlCompute;
-    if (fl & kFlNonFinite) record_error(err, CS_ERR_NONFINITE);
-    if (fl & kFlArg) record_error(err, CS_ERR_ARG);
-    s_flag[i] = fl;
-    accum[i] = a;
-    skip_mask[i] = compute ? 0 : 1;
-    has_ref[i] = compute ? 1 : 3;
-  }
-  block_sync();
-  if (warp == 0) {
-    int nc = 0;
-    for (int base = 0; base < N; base += 32) {
-      const int k = base + lane;
-      const bool comp = k < N && (s_flag[k] & kFlCompute);
-      const unsigned b = __ballot_sync(0xffffffffu, comp);
-      if (comp) idx[nc + __popc(b & ((1u << lane) - 1u))] = k;
-      nc += __popc(b);
+  if constexpr (kDecide) {   // the state writes of the deciding form
+    for (int i = threadIdx.x; i < N; i += kSkipThreads) {
+      float a;
+      const uint8_t fl = decide_carried(i, wf, tau, has_ref, accum, drift_in, force, a);
+      const bool compute = fl & kFlCompute;
+      if (fl & kFlNonFinite) record_error(err, CS_ERR_NONFINITE);
+      if (fl & kFlArg) record_error(err, CS_ERR_ARG);
+      s_flag[i] = fl;
+      accum[i] = a;
+      skip_mask[i] = compute ? 0 : 1;
+      has_ref[i] = compute ? 1 : 3;
     }
-    if (lane == 0) *n_compute = nc;
+    block_sync();
+    if (warp == 0) {
+      int nc = 0;
+      for (int base = 0; base < N; base += 32) {
+        const int k = base + lane;
+        const bool comp = k < N && (s_flag[k] & kFlCompute);
+        const unsigned b = __ballot_sync(0xffffffffu, comp);
+        if (comp) idx[nc + __popc(b & ((1u << lane) - 1u))] = k;
+        nc += __popc(b);
+      }
+      if (lane == 0) *n_compute = nc;
+    }
   }
 }
 
