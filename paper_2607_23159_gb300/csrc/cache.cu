@@ -882,9 +882,11 @@ __global__ void __launch_bounds__(kSkipThreads, 1) carry_skip_kernel(
     if (lane == 0 && items > 0)
       for (int j = 0; j < S && !exhausted; ++j) fill(j);
     n_real = __shfl_sync(0xffffffffu, n_real, 0);
+    int j_released = 0;                            // uses whose copies have landed and been consumed
     for (int j = 0; j < n_real; ++j) {
       const int st = j % S;
       if (!mbar_wait(&empty[st], (uint32_t)(j / S) & 1u, abort, err)) break;   // the consumers are done with use j
+      j_released = j + 1;
       if (lane == 0) {
         const int it = s_item[st], sq = it / nun, u = it - sq * nun, i = s_list[sq];
         float p[NV];
@@ -901,8 +903,9 @@ __global__ void __launch_bounds__(kSkipThreads, 1) carry_skip_kernel(
       n_real = __shfl_sync(0xffffffffu, n_real, 0);
     }
     if (*abort && lane == 0) {
-      // a wait ran out: let every copy this CTA issued land before its memory goes
-      for (int j = 0; j < n_real; ++j) mbar_wait_teardown(&full[j % S], (uint32_t)(j / S) & 1u);
+      // a wait ran out: let the copies still outstanding (uses not yet released) land
+      // before the CTA's memory goes
+      for (int j = j_released; j < n_real; ++j) mbar_wait_teardown(&full[j % S], (uint32_t)(j / S) & 1u);
     }
     if (lane == 0) {
       // the claims made ahead must be performed before this CTA arrives (the last CTA to
@@ -1575,6 +1578,10 @@ cs_status carry_decide_skip_run(float* x, const float* x_ref, const float* delta
   const float2* din = reinterpret_cast<const float2*>(b + L.drift) + (size_t)(step_k & 1) * cs.cap;
   float* spart = reinterpret_cast<float*>(b + L.spart);
   const int nch = L.nch, nun = L.nun;
+  if ((long long)N * nun >= (1ll << 31) || N > 4096) {
+    set_error("carry_decide_skip_run: %d candidates of %lld elements exceed the item range", N, D);
+    return CS_ERR_UNSUPPORTED;
+  }
   const float h = t_next - t_cur;
   const size_t smem = carry_skip_smem(N);
   int grid = num_sms();                           // one CTA per SM (the ring takes its shared memory)
