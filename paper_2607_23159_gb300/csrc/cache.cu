@@ -843,7 +843,10 @@ __global__ void __launch_bounds__(kSkipThreads, 1) carry_skip_kernel(
     // them through L2 (a read-only cached load could be placed before the wait)
     pdl_wait_primary();
     ns = __ldcg(sidx_in + N);
-    for (int q = threadIdx.x; q < ns; q += kSkipThreads) s_list[q] = (uint16_t)__ldcg(sidx_in + q);
+    for (int q = threadIdx.x; q < ns; q += kSkipThreads) {
+      const int i = __ldcg(sidx_in + q);
+      s_list[q] = (uint16_t)(index_ok(i, N, err) ? i : 0);   // checked in CS_DEBUG_CHECKS builds
+    }
     block_sync();
   }
   const int items = ns * nun;
